@@ -1,0 +1,453 @@
+"""Benchmark of the cached-reference joint attention on one GB300 (or N replicas).
+
+One timed step = one layer's whole hot path for one generation of the
+1024x1024, five-reference edit: refcache_build (cache write + [ST; R] prefill)
+followed by T = 40 step_attention calls with fresh live Q/K/V each denoising
+step (four live input sets cycled, so every step streams more than the 129 MB
+L2: 252 MB of cache plus 85 MB of live Q/K/V).  `value` is the unmasked
+TFLOP/s of that step (4 d FLOPs per visible (query, key) pair per head).
+
+Also reported: the step-attention kernel alone (ms per call, TFLOP/s, its
+roofline against the measured bf16 peak), the prefill alone, the
+full-attention recompute on the same kernel, the measured and modelled
+40-step speedups, an end-to-end number through the C ABI with host buffers,
+SM clocks sampled during the timed region, and the CPU oracle timed on a
+bounded sample (the reported CPU baseline).
+
+`--impl reference` times the CPU oracle instead (this workload has no other
+reference implementation), on bounded samples of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "cached-ref attention TFLOP/s & ms/step (5 refs,1024²); modelled 40-step speedup"
+UNIT = "TFLOP/s"
+T_STEPS = 40
+N_LIVE_SETS = 4
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {"bf16_burst": float(p["bf16_tflops"]), "bf16_sustained": float(p["bf16_tflops_sustained"]),
+                "hbm_gbs": float(p["hbm_gbs"]), "source": "measured"}
+    except Exception:
+        return {"bf16_burst": 1900.0, "bf16_sustained": 1700.0, "hbm_gbs": 6800.0, "source": "fallback"}
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.tmp = None
+
+    def __enter__(self):
+        try:
+            self.tmp = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=self.tmp, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+        return False
+
+    def summary(self):
+        if self.proc is None or self.tmp is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.tmp.flush()
+        rows = []
+        with open(self.tmp.name) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.tmp.name)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        mx = [num(r[2]) for r in rows if num(r[2]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower() == "active"})
+        loaded = [s for s in sm if s > 0.5 * max(sm)] if sm else []
+        return {"sm_mhz": statistics.median(loaded) if loaded else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows),
+                "power_w_max": max((num(r[3]) or 0.0) for r in rows)}
+
+
+# ----------------------------------------------------------------------------- distributed
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def aggregate(local_flops: float, local_seconds: float, world_size: int):
+    """Whole-job throughput of weakly scaled replicas: every rank's work over
+    the slowest rank's time (max over ranks), as the contract requires."""
+    if world_size == 1:
+        return local_flops, local_seconds
+    import torch
+    import torch.distributed as dist
+
+    dev = torch.device("cuda", torch.cuda.current_device()) if dist.get_backend() == "nccl" else torch.device("cpu")
+    t = torch.tensor([local_seconds], dtype=torch.float64, device=dev)
+    f = torch.tensor([local_flops], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(f, op=dist.ReduceOp.SUM)
+    return float(f.item()), float(t.item())
+
+
+# ----------------------------------------------------------------------------- our arm
+def run_ours(args, ws, rank, local):
+    import torch
+
+    import workloads
+    from paper_2608_21229_gb300 import accounting as acc
+    from paper_2608_21229_gb300 import build as cbuild
+    from paper_2608_21229_gb300 import refcache as rcb
+
+    cbuild.build()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    rcb.set_kernel(args.kernel)
+    w = workloads.ALL[args.workload]
+    H, D = w.num_heads, w.head_dim
+    seg = rcb.Segments.from_workload(w)
+    cache = rcb.RefCache(seg, num_layers=1, mask_mode="beyond", device=dev)
+    scale = 1.0 / math.sqrt(D)
+    qs, ks, vs = (t.to(dev) for t in workloads.static_qkv(w))
+    lives = [tuple(t.to(dev) for t in workloads.live_qkv(w, step=i)) for i in range(N_LIVE_SETS)]
+    o_s = torch.empty(seg.static_rows, H, D, dtype=torch.bfloat16, device=dev)
+    o_l = torch.empty(seg.live_rows, H, D, dtype=torch.bfloat16, device=dev)
+    stream = torch.cuda.current_stream()
+
+    pre_flops = acc.flops(acc.prefill_units(w.requests), H, D)
+    step_flops = acc.flops(acc.step_units(w.requests), H, D)
+    full_flops = acc.flops(acc.full_units(w.requests), H, D)
+    flops_per_step = pre_flops + T_STEPS * step_flops
+    launches_per_step = (1 if acc.cache_bytes(w.requests, H, D) else 0) + 1 + T_STEPS
+
+    def one_step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        cache.build(0, qs, ks, vs, o_s, scale=scale)
+        if ev is not None:
+            ev[1].record(stream)
+        for t in range(T_STEPS):
+            ql, kl, vl = lives[t % N_LIVE_SETS]
+            cache.step(0, ql, kl, vl, o_l, scale=scale)
+            if ev is not None:
+                ev[2 + t].record(stream)
+
+    for _ in range(args.warmup):
+        one_step()
+    torch.cuda.synchronize()
+    st = rcb.status()
+    if st != rcb.OK:
+        raise RuntimeError(f"device error during warm-up: {rcb.last_error()}")
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2 + T_STEPS)] for _ in range(args.steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if ws > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        start.record(stream)
+        for k in range(args.steps):
+            one_step(evs[k])
+        end.record(stream)
+        torch.cuda.synchronize()
+    if ws > 1:
+        dist.barrier()
+    if rcb.status() != rcb.OK:
+        raise RuntimeError(f"device error in the timed region: {rcb.last_error()}")
+    total_s = start.elapsed_time(end) / 1e3
+    pre_ms = [e[0].elapsed_time(e[1]) for e in evs]
+    step_ms = [e[1 + t].elapsed_time(e[2 + t]) for e in evs for t in range(T_STEPS)]
+    t_pre = statistics.mean(pre_ms) / 1e3
+    t_step = statistics.mean(step_ms) / 1e3
+
+    # full-attention recompute of the same request on the same kernel (baseline, not timed above)
+    r = w.requests[0]
+    n_full = sum(x.n_lt + x.n_x + x.n_r for x in w.requests)
+    cu_full = [0]
+    for x in w.requests:
+        cu_full.append(cu_full[-1] + x.n_lt + x.n_x + x.n_r)
+    qf, kf, vf = (workloads.randn_bf16((n_full, H, D), w.seed, f"full_{c}").to(dev) for c in "qkv")
+    o_f = torch.empty(n_full, H, D, dtype=torch.bfloat16, device=dev)
+    for _ in range(2):
+        rcb.full_attention(cu_full, qf, kf, vf, o_f, scale=scale)
+    fe = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    fe[0].record(stream)
+    for i in range(3):
+        rcb.full_attention(cu_full, qf, kf, vf, o_f, scale=scale)
+    fe[1].record(stream)
+    torch.cuda.synchronize()
+    t_full = fe[0].elapsed_time(fe[1]) / 3e3
+    del qf, kf, vf, o_f
+
+    e2e = run_e2e(args, w, cache, seg, dev, stream, scale, flops_per_step)
+    flops_all, secs_all = aggregate(flops_per_step * args.steps, total_s, ws)
+    pk = peaks()
+    achieved = step_flops / t_step / 1e12
+    line = {
+        "metric": METRIC,
+        "value": flops_all / secs_all / 1e12,
+        "unit": UNIT,
+        "n_gpus": ws,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": secs_all / args.steps * 1e3,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic",
+        "config": {
+            "workload": w.name, "num_heads": H, "head_dim": D,
+            "requests": [[x.n_st, x.n_lt, x.n_x, x.n_r] for x in w.requests],
+            "segments": "(N_ST, N_LT, N_X, N_R) per request",
+            "step": f"refcache_build + {T_STEPS} step_attention (one layer, one generation)",
+            "mask": "beyond (Sec. 3.3)", "kernel": args.kernel,
+            "l2": f"inputs larger than L2: {acc.cache_bytes(w.requests, H, D) / 1e6:.0f} MB cache + "
+                  f"{N_LIVE_SETS} live Q/K/V sets of {3 * seg.live_rows * H * D * 2 / 1e6:.0f} MB cycled",
+            "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU",
+        },
+        "step_attention": {"ms": t_step * 1e3, "tflops": achieved, "flops": step_flops},
+        "prefill": {"ms": t_pre * 1e3, "tflops": pre_flops / t_pre / 1e12, "flops": pre_flops},
+        "full_attention": {"ms": t_full * 1e3, "tflops": full_flops / t_full / 1e12, "flops": full_flops},
+        "speedup_40step": {
+            "measured": acc.measured_ratio(t_full, t_pre, t_step, T_STEPS),
+            "interaction_model": acc.modelled_ratio(w.requests, T_STEPS),
+            "paper_end_to_end": {"5_refs": 3.92, "10_refs": 5.47, "note": "whole model, unnamed GPU (context)"},
+        },
+        "roofline": {
+            "kernel": f"attn_{args.kernel}_kernel<{D}> (step_attention)",
+            "bound": "tensor", "achieved": achieved, "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
+            "frac": achieved / pk["bf16_sustained"],
+            "peak_kind": f"bf16 dense, {pk['source']} sustained (kernel timed inside a long step)",
+            "frac_of_burst": achieved / pk["bf16_burst"],
+            "traffic": None,
+            "algorithmic_bytes": 2 * (seg.live_rows * H * D * 2) * 2 + acc.cache_bytes(w.requests, H, D),
+        },
+        "e2e": e2e,
+        "clocks": clk.summary(),
+        "gpu_launches": launches_per_step * args.steps,
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget)
+    return line
+
+
+def run_e2e(args, w, cache, seg, dev, stream, scale, flops_per_step):
+    """The same step through the public API with host buffers: pinned host
+    inputs copied in and outputs copied back inside the timed region."""
+    import torch
+
+    import workloads
+
+    H, D = w.num_heads, w.head_dim
+    hs = [t.pin_memory() for t in workloads.static_qkv(w)]
+    hl = [[t.pin_memory() for t in workloads.live_qkv(w, step=i)] for i in range(N_LIVE_SETS)]
+    ds = [torch.empty_like(t, device=dev) for t in hs]
+    dl = [torch.empty_like(t, device=dev) for t in hl[0]]
+    o_s = torch.empty(seg.static_rows, H, D, dtype=torch.bfloat16, device=dev)
+    o_l = torch.empty(seg.live_rows, H, D, dtype=torch.bfloat16, device=dev)
+    ho_s = torch.empty(o_s.shape, dtype=torch.bfloat16).pin_memory()
+    ho_l = torch.empty(o_l.shape, dtype=torch.bfloat16).pin_memory()
+    h2d = sum(t.numel() * 2 for t in hs) + T_STEPS * sum(t.numel() * 2 for t in hl[0])
+    d2h = ho_s.numel() * 2 + T_STEPS * ho_l.numel() * 2
+
+    def one():
+        for d, h in zip(ds, hs):
+            d.copy_(h, non_blocking=True)
+        cache.build(0, ds[0], ds[1], ds[2], o_s, scale=scale)
+        ho_s.copy_(o_s, non_blocking=True)
+        for t in range(T_STEPS):
+            for d, h in zip(dl, hl[t % N_LIVE_SETS]):
+                d.copy_(h, non_blocking=True)
+            cache.step(0, dl[0], dl[1], dl[2], o_l, scale=scale)
+            ho_l.copy_(o_l, non_blocking=True)
+
+    one()
+    torch.cuda.synchronize()
+    n = max(1, min(args.steps, 3))
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(n):
+        one()
+    b.record(stream)
+    torch.cuda.synchronize()
+    secs = a.elapsed_time(b) / 1e3 / n
+    return {"value": flops_per_step / secs / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "ms_per_step": secs * 1e3, "steps": n}
+
+
+# ----------------------------------------------------------------------------- CPU oracle
+def oracle_sample(w, n_pairs_step, n_pairs_pre, seed=0):
+    """A bounded sample of the workload for the CPU oracle: (row, head) pairs of
+    the step and of the prefill, in proportion to their share of the FLOPs."""
+    import numpy as np
+
+    import workloads
+
+    rng = np.random.default_rng(seed)
+    r = w.requests[0]
+    static = [workloads.bf16_bits(t) for t in workloads.static_qkv(w)]
+    live = [workloads.bf16_bits(t) for t in workloads.live_qkv(w)]
+    sp = np.stack([rng.integers(0, r.n_live, n_pairs_step), rng.integers(0, w.num_heads, n_pairs_step)], 1)
+    pp = np.stack([rng.integers(0, r.n_static, n_pairs_pre), rng.integers(0, w.num_heads, n_pairs_pre)], 1)
+    return static, live, sp.astype(np.int32), pp.astype(np.int32)
+
+
+def time_oracle_sample(w, static, live, sp, pp):
+    """Time the oracle's attention on the sampled outputs (the joint sequences
+    are assembled before the clock starts)."""
+    import oracle
+
+    r = w.requests[0]
+    scale = 1.0 / math.sqrt(w.head_dim)
+    kc, vc = oracle.cached_kv(static[1], static[2], r.n_st, "beyond")
+    joint = oracle.step_inputs(*live, kc, vc, r.n_lt, r.n_x, r.n_st, r.n_r, "beyond")
+    t0 = time.perf_counter()
+    oracle.joint_attention(*static, 0, 0, r.n_st, r.n_r, "beyond", scale, pp)
+    oracle.joint_attention(*joint, r.n_lt, r.n_x, r.n_st, r.n_r, "beyond", scale, sp)
+    secs = time.perf_counter() - t0
+    d = w.head_dim
+    flops = 4 * d * (len(sp) * (r.n_live + r.n_r) + len(pp) * (r.n_st + r.n_r))
+    return flops, secs
+
+
+def sample_sizes(w, total_pairs):
+    from paper_2608_21229_gb300 import accounting as acc
+
+    r = w.requests[0]
+    pre = acc.prefill_units(w.requests)
+    stp = T_STEPS * acc.step_units(w.requests)
+    # a step pair costs (N_live + N_R) units, a prefill pair (N_ST + N_R): keep
+    # the sample's prefill/step FLOP ratio equal to the workload's
+    n_step = max(1, int(total_pairs))
+    n_pre = max(1, round(n_step * (pre / stp) * (r.n_live + r.n_r) / (r.n_st + r.n_r)))
+    return n_step, n_pre
+
+
+def cpu_baseline(w, budget_s=15.0):
+    import oracle
+
+    oracle.build()
+    static, live, sp, pp = oracle_sample(w, *sample_sizes(w, 64))
+    f, s = time_oracle_sample(w, static, live, sp, pp)  # calibration
+    scale = max(1.0, budget_s / max(s, 1e-3))
+    n_step, n_pre = sample_sizes(w, int(64 * scale))
+    static, live, sp, pp = oracle_sample(w, n_step, n_pre, seed=1)
+    f, s = time_oracle_sample(w, static, live, sp, pp)
+    return {"value": f / s / 1e12, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+            "sample": f"{len(sp)} (row, head) outputs of the step and {len(pp)} of the prefill of {w.name}, "
+                      f"fp64 plain definition, {s:.1f} s",
+            "seconds": s, "flops": f}
+
+
+def run_reference(args, ws, rank):
+    if rank != 0:
+        return None
+    import oracle
+
+    import workloads
+
+    oracle.build()
+    w = workloads.ALL[args.workload]
+    n_step, n_pre = sample_sizes(w, args.ref_pairs)
+    static, live, sp, pp = oracle_sample(w, n_step, n_pre)
+    for _ in range(args.warmup):
+        time_oracle_sample(w, static, live, sp[:8], pp[:1])
+    tot_f = tot_s = 0.0
+    for _ in range(args.steps):
+        f, s = time_oracle_sample(w, static, live, sp, pp)
+        tot_f += f
+        tot_s += s
+    v = tot_f / tot_s / 1e12
+    sample = f"per step {len(sp)} step and {len(pp)} prefill (row, head) outputs of {w.name}"
+    return {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": tot_s / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": w.name, "note": "CPU oracle (plain fp64 definition) on bounded samples"},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="edit1024_5ref")
+    ap.add_argument("--kernel", choices=["tcgen05", "mma_sync"], default="tcgen05")
+    ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
+    ap.add_argument("--ref-pairs", type=int, default=192, help="oracle (row, head) outputs per reference step")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    ws, rank, local = dist_env()
+    if args.warmup < 3:
+        args.warmup = 3
+    if ws > 1 and args.impl == "ours":
+        import torch
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    if args.impl == "reference":
+        line = run_reference(args, ws, rank)
+    else:
+        line = run_ours(args, ws, rank, local)
+    if rank == 0 and line is not None:
+        print(json.dumps(line), flush=True)
+    if ws > 1 and args.impl == "ours":
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,209 @@
+/*
+ * refcache.h -- C ABI of the beyond-mask joint attention library for GB300
+ * (sm_103a): exact reference K/V caching with static text anchors.
+ *
+ * The paper's method (Sec. 3.3 "Static Text Anchors", App. C "Derivation"):
+ * one request's in-context sequence is [LT, X_t, ST, R] -- live instruction
+ * text, the denoising target, static text anchors (the instruction embedded
+ * once at t = 0) and the tokens of K reference images R = [R(1); ...; R(K)]
+ * (Eq. 1).  R and ST attend each other and nothing else, so their layerwise
+ * K and V (Eq. 2) never depend on X_t and are computed once; the live rows
+ * [LT, X_t] attend [LT, X_t, R] at every denoising step.
+ *
+ *   refcache_build   the one-shot static prefill: rows [ST; R] attend keys
+ *                    [ST; R]; the R rows' K and V are written into the
+ *                    persistent per-layer cache (Sec. 3.3, Eq. cost-pre).
+ *   step_attention   one layer of one denoising step: rows [LT; X_t] attend
+ *                    their own keys and the cached R keys (App. C, Eq.
+ *                    cost-step); no mask is materialised.
+ *   full_attention   the full-attention recompute every key of [LT; X_t; R]
+ *                    visible to every row (Sec. 3.2, C_full in App. C): the
+ *                    baseline the cache is measured against.
+ *
+ * Conventions shared by every entry point
+ *   - Tensors are THD: [tokens, num_heads, head_dim] bf16, head_dim
+ *     contiguous, rows of consecutive requests packed back to back.  Base
+ *     pointers must be device pointers aligned to 16 bytes.
+ *   - head_dim is 64 or 128; num_heads >= 1.
+ *   - Every input row must hold finite values (rows of a neighbouring request
+ *     may be read into a tile and masked out; they must not be NaN/Inf).
+ *   - softmax_scale must be finite and > 0 (1/sqrt(head_dim) is the usual
+ *     choice; the paper does not state it).
+ *   - lse outputs are optional (NULL = not written): fp32 [tokens, num_heads],
+ *     natural-log log-sum-exp of the scaled scores of each row.
+ *   - Outputs are bf16 rounded to nearest-even; scores, softmax and
+ *     accumulation are fp32; P is rounded to bf16 before the P.V product.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t passed as void*;
+ *     NULL = legacy default stream) and return a status code below.  A
+ *     non-zero return means nothing was launched.  Device-side faults of a
+ *     launched kernel (a bounded wait that ran out) are reported later by
+ *     refcache_status().
+ *   - Host arrays (segment tables) are read during the call only; the library
+ *     keeps its own copies.
+ *   - No entry point allocates device memory except refcache_create (unless it
+ *     is given memory) and full_attention (a per-device work-list buffer that
+ *     it keeps and grows).
+ */
+#ifndef REFCACHE_H
+#define REFCACHE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define REFCACHE_API __attribute__((visibility("default")))
+#else
+#define REFCACHE_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ------------------------------------------------------ */
+#define REFCACHE_OK 0
+#define REFCACHE_ERR_INVALID_ARG (-1) /* null/misaligned pointer, bad sizes or offsets */
+#define REFCACHE_ERR_UNSUPPORTED (-2) /* head_dim not 64/128, no sm_103 device */
+#define REFCACHE_ERR_NOT_BUILT (-3)   /* step_attention on a layer whose cache was not built */
+#define REFCACHE_ERR_CUDA (-4)        /* a CUDA runtime/driver call failed */
+#define REFCACHE_ERR_OOM (-5)         /* device allocation failed or given memory too small */
+#define REFCACHE_ERR_TIMEOUT (-6)     /* a kernel's bounded wait ran out (see refcache_status) */
+
+/* ---- mask modes (who the static rows and the live rows attend) ---------- */
+/* Sec. 3.3: ST <-> R both ways, live rows attend [LT, X_t, R], not ST.      */
+#define REFCACHE_MASK_BEYOND 0
+/* Alternative anchor reading: ST rows attend only ST, R rows attend [ST, R],
+ * live rows attend [LT, X_t, ST, R]; the cache then keeps ST's K/V too.     */
+#define REFCACHE_MASK_BEYOND_ALT 1
+/* Sec. 4.1 isolated cache (prior-art topology): R attends only R; every
+ * request must have zero anchors.                                            */
+#define REFCACHE_MASK_ISOLATED 2
+
+/* Kernel selection (refcache_set_kernel): the tcgen05/TMEM/TMA kernel is the
+ * default; the mma.sync kernel is the recompiled legacy-tensor-core baseline. */
+#define REFCACHE_KERNEL_TCGEN05 0
+#define REFCACHE_KERNEL_MMA_SYNC 1
+
+/*
+ * Segment table of a batch of requests (Eq. 1 layout, Sec. 3.3 order).
+ * All arrays are HOST memory.
+ *   cu_live[batch+1]   offsets of each request's [LT; X_t] rows in the step
+ *                      tensors (cu_seqlens style, cu_live[0] = 0, non-decreasing)
+ *   cu_static[batch+1] offsets of each request's [ST; R] rows in the prefill
+ *                      tensors
+ *   n_anchor[batch]    N_ST: the first n_anchor[b] rows of request b's static
+ *                      segment are anchors, the rest are R (N_R >= 0)
+ *   n_instr[batch]     N_LT (may be NULL): the first rows of each live segment
+ *                      are instruction text; LT and X_t are attended alike, so
+ *                      it is informational
+ */
+typedef struct {
+  int32_t batch;
+  int32_t num_heads;
+  int32_t head_dim;
+  const int32_t* cu_live;
+  const int32_t* cu_static;
+  const int32_t* n_anchor;
+  const int32_t* n_instr;
+} refcache_segments_t;
+
+typedef struct refcache refcache_t; /* opaque; owns the per-layer K/V slots */
+
+/*
+ * Device bytes a cache needs for `num_layers` layers (Sec. 3.3: per layer the
+ * R rows' K and V, bf16, [cache_rows, num_heads, head_dim] each, plus the
+ * anchors' rows in REFCACHE_MASK_BEYOND_ALT), plus its small work tables.
+ * Returns 0 for invalid arguments.
+ */
+REFCACHE_API size_t refcache_bytes(int num_layers, int mask_mode, const refcache_segments_t* seg);
+
+/*
+ * Create a cache.  If dev_mem is NULL the library allocates refcache_bytes()
+ * with cudaMalloc on the current device and frees it in refcache_destroy;
+ * otherwise it uses dev_mem (>= refcache_bytes(), 256-byte aligned, owned by
+ * the caller, not freed).  Synchronous.  *out is set only on success.
+ */
+REFCACHE_API int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refcache_segments_t* seg,
+                    void* dev_mem, size_t dev_bytes);
+
+/* Free the cache (waits for the device to finish using it).  NULL is a no-op. */
+REFCACHE_API void refcache_destroy(refcache_t* cache);
+
+/*
+ * Device pointers of layer `layer`'s K and V slots, each a THD bf16 tensor of
+ * *rows rows: request b's cached rows follow request b-1's.  Cached rows are
+ * R (Eq. 2), or [ST; R] in REFCACHE_MASK_BEYOND_ALT.  Any output may be NULL.
+ */
+REFCACHE_API int refcache_kv_ptr(refcache_t* cache, int layer, void** k_slot, void** v_slot, int64_t* rows);
+
+/* 1 if `layer` has been built, 0 if not, < 0 on error. */
+REFCACHE_API int refcache_layer_built(refcache_t* cache, int layer);
+
+/*
+ * Static prefill of one layer (Sec. 3.3; cost (N_R + N_ST)^2 per head,
+ * Eq. cost-pre).  q_static/k_static/v_static: [cu_static[batch], H, d] bf16,
+ * each request's [ST; R] rows.  Writes o_static (same shape) for every ST and
+ * R row, lse_static if non-NULL, and copies the cached rows' K and V into the
+ * layer's slots.  The result does not depend on any live input, and repeated
+ * builds with the same inputs produce the same bytes.
+ */
+REFCACHE_API int refcache_build(refcache_t* cache, int layer, const void* q_static, const void* k_static,
+                   const void* v_static, void* o_static, float* lse_static, float softmax_scale,
+                   void* stream);
+
+/*
+ * One denoising step of one layer (App. C: [LT, X_t] queries over
+ * [LT, X_t, R]; cost S (N_R + S) per head, Eq. cost-step).  q_live, k_live,
+ * v_live: [cu_live[batch], H, d] bf16, each request's [LT; X_t] rows.  Keys
+ * are the request's own live rows followed by its cached rows of `layer`.
+ * Writes o_live (same shape) and lse_live if non-NULL.
+ * Returns REFCACHE_ERR_NOT_BUILT if the layer was never built.
+ */
+REFCACHE_API int step_attention(refcache_t* cache, int layer, const void* q_live, const void* k_live,
+                   const void* v_live, void* o_live, float* lse_live, float softmax_scale,
+                   void* stream);
+
+/*
+ * Full attention (Sec. 3.2; C_full = T (N_R + S)^2 over T steps, App. C):
+ * every row of request b attends every key of request b.  cu_seqlens is a
+ * HOST array [batch+1]; q, k, v, o are [cu_seqlens[batch], H, d] bf16.
+ * Uses (and on first use or growth allocates) a per-device work-list buffer
+ * kept by the library; calls on one device must be ordered on one stream.
+ */
+REFCACHE_API int full_attention(int batch, int num_heads, int head_dim, const int32_t* cu_seqlens, const void* q,
+                   const void* k, const void* v, void* o, float* lse, float softmax_scale,
+                   void* stream);
+
+/*
+ * Synchronise `stream`, then read and clear the current device's error word
+ * written by kernels whose bounded waits ran out.  Returns REFCACHE_OK,
+ * REFCACHE_ERR_TIMEOUT or REFCACHE_ERR_CUDA.
+ */
+REFCACHE_API int refcache_status(void* stream);
+
+/* Wait limit of every in-kernel wait, nanoseconds (default 1e9).  Returns the old value. */
+REFCACHE_API uint64_t refcache_set_wait_timeout_ns(uint64_t ns);
+
+/* Select the kernel for subsequent calls (REFCACHE_KERNEL_*); returns the old one or < 0. */
+REFCACHE_API int refcache_set_kernel(int kernel);
+
+/*
+ * Debug fault injection on the host side of the wait protocol: when `on` is
+ * non-zero, the next launch's TMA producer skips its first K-tile load, so
+ * the consumers' bounded waits run out and the kernel reports
+ * REFCACHE_ERR_TIMEOUT through refcache_status() instead of hanging.  The
+ * switch clears itself after one launch.  Only the tcgen05 kernel has it.
+ */
+REFCACHE_API void refcache_debug_skip_first_load(int on);
+
+/* Copy the calling thread's last error message into buf (NUL-terminated); returns its length. */
+REFCACHE_API int refcache_last_error(char* buf, size_t n);
+
+/* Library version string. */
+REFCACHE_API const char* refcache_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* REFCACHE_H */

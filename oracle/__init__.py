@@ -146,6 +146,8 @@ def joint_attention(q, k, v, n_lt, n_x, n_st, n_r, mode, scale, pairs=None):
         npairs = pairs.shape[0]
         out = np.zeros((npairs, d), np.float64)
         lse = np.zeros((npairs,), np.float64)
+        if npairs == 0:
+            return out, lse
         pp = _ptr(pairs, ctypes.c_int32)
     rc = lib().oracle_joint_attention(
         _ptr(q, ctypes.c_uint16), _ptr(k, ctypes.c_uint16), _ptr(v, ctypes.c_uint16),
@@ -165,22 +167,26 @@ def prefill(q_s, k_s, v_s, n_st, n_r, mode, scale, pairs=None):
     the cache also keeps the anchors' K and V, so it is the whole [ST; R].
     """
     out, lse = joint_attention(q_s, k_s, v_s, 0, 0, n_st, n_r, mode, scale, pairs)
+    k_c, v_c = cached_kv(k_s, v_s, n_st, mode)
+    return out, lse, k_c, v_c
+
+
+def cached_kv(k_s, v_s, n_st, mode):
+    """What the static pass keeps (Sec. 3.3): the R rows' K and V, Eq. 2 -- plus
+    the anchors' rows in the alternative anchor reading."""
     keep = 0 if mode == "beyond_alt" else n_st
-    return out, lse, np.array(k_s[keep:], copy=True), np.array(v_s[keep:], copy=True)
+    return np.array(k_s[keep:], copy=True), np.array(v_s[keep:], copy=True)
 
 
-def step(q_l, k_l, v_l, k_cache, v_cache, n_lt, n_x, n_st, n_r, mode, scale, pairs=None):
-    """One denoising step for one request (App. C "Derivation").
-
-    The live rows [LT; X_t] query the joint sequence whose ST/R keys come from
-    the cache.  ``k_cache``/``v_cache`` hold R (or [ST; R] in the alternative
-    anchor reading).  Rows of ST and R are not computed; their queries are
-    zero placeholders.  Returns (out, lse) for the live rows.
-    """
+def step_inputs(q_l, k_l, v_l, k_cache, v_cache, n_lt, n_x, n_st, n_r, mode):
+    """The joint sequence [LT; X_t; ST; R] of one denoising step (Sec. 3.3
+    order), with the ST/R keys and values taken from the cache.  Queries of the
+    ST and R rows are zero placeholders (those rows are not computed in a
+    step); in the paper's mask the anchors' K/V are not cached and not
+    visible to live rows, so their slots hold zeros."""
     q_l, k_l, v_l = _u16(q_l), _u16(k_l), _u16(v_l)
     H, d = q_l.shape[1:]
-    n_live = n_lt + n_x
-    assert q_l.shape[0] == n_live
+    assert q_l.shape[0] == n_lt + n_x
     if mode == "beyond_alt":
         assert k_cache.shape[0] == n_st + n_r
         k_st, v_st = k_cache[:n_st], v_cache[:n_st]
@@ -193,8 +199,22 @@ def step(q_l, k_l, v_l, k_cache, v_cache, n_lt, n_x, n_st, n_r, mode, scale, pai
     q = np.concatenate([q_l, np.zeros((n_st + n_r, H, d), np.uint16)])
     k = np.concatenate([k_l, k_st, k_r])
     v = np.concatenate([v_l, v_st, v_r])
+    return q, k, v
+
+
+def step(q_l, k_l, v_l, k_cache, v_cache, n_lt, n_x, n_st, n_r, mode, scale, pairs=None):
+    """One denoising step for one request (App. C "Derivation").
+
+    The live rows [LT; X_t] query the joint sequence whose ST/R keys come from
+    the cache (``step_inputs``).  ``k_cache``/``v_cache`` hold R (or [ST; R] in
+    the alternative anchor reading).  Returns (out, lse) of the live rows:
+    [n_live, H, d] / [n_live, H], or per pair with ``pairs``.
+    """
+    q, k, v = step_inputs(q_l, k_l, v_l, k_cache, v_cache, n_lt, n_x, n_st, n_r, mode)
+    H, d = q.shape[1:]
+    n_live = n_lt + n_x
     if pairs is None:
-        pairs = np.array([(i, h) for i in range(n_live) for h in range(H)], np.int32)
+        pairs = np.array([(i, h) for i in range(n_live) for h in range(H)], np.int32).reshape(-1, 2)
         out, lse = joint_attention(q, k, v, n_lt, n_x, n_st, n_r, mode, scale, pairs)
         return out.reshape(n_live, H, d), lse.reshape(n_live, H)
     pairs = np.asarray(pairs, np.int32).reshape(-1, 2)

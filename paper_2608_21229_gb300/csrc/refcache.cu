@@ -1,0 +1,613 @@
+// refcache.cu -- the C ABI declared in include/refcache.h: argument checks,
+// the per-request work tables, the persistent per-layer K/V cache, TMA tensor
+// maps and the kernel launches.  All compute runs in the kernels of
+// attn_tc.cuh (default) or attn_mma.cuh.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "refcache.h"
+#include "attn_mma.cuh"
+#include "attn_tc.cuh"
+
+using rc::AttnArgs;
+using rc::CopySeg;
+using rc::Task;
+
+namespace {
+
+thread_local std::string g_last_error;
+std::atomic<int> g_kernel{REFCACHE_KERNEL_TCGEN05};
+std::atomic<uint64_t> g_timeout_ns{1000000000ull};
+std::atomic<int> g_dbg_skip{0};
+
+int fail(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return code;
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+  return fail(REFCACHE_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+constexpr int kMaxDevices = 64;
+
+struct DeviceInfo {
+  bool checked = false;
+  bool ok = false;
+  int num_sms = 0;
+  bool attr_set[4] = {false, false, false, false};
+};
+DeviceInfo g_dev[kMaxDevices];
+std::mutex g_dev_mu;
+
+// The kernels are built for sm_103a only: require a compute capability 10.3 device.
+int current_device(int* dev_out, DeviceInfo** info) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return fail(REFCACHE_ERR_UNSUPPORTED, "device index %d", dev);
+  std::lock_guard<std::mutex> lk(g_dev_mu);
+  DeviceInfo& d = g_dev[dev];
+  if (!d.checked) {
+    int major = 0, minor = 0, sms = 0;
+    if ((e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+      return cuda_fail(e, "cudaDeviceGetAttribute");
+    d.checked = true;
+    d.ok = (major == 10 && minor == 3);
+    d.num_sms = sms;
+    if (!d.ok) {
+      d.checked = false;
+      return fail(REFCACHE_ERR_UNSUPPORTED, "device %d is sm_%d%d; this library is built for sm_103a", dev,
+                  major, minor);
+    }
+  }
+  *dev_out = dev;
+  *info = &d;
+  return REFCACHE_OK;
+}
+
+// ---------------------------------------------------------------- tensor maps
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// THD bf16 tensor [rows, H, D] seen as a 2-D array (H*D columns, rows rows);
+// box = 64 columns (128 bytes) x 128 rows with the 128-byte swizzle.
+int make_tmap(CUtensorMap* m, const void* base, int64_t rows, int H, int D) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return fail(REFCACHE_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(H) * D, static_cast<cuuint64_t>(std::max<int64_t>(rows, 1))};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(H) * D * 2};
+  const cuuint32_t box[2] = {64, 128};
+  const cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(REFCACHE_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
+  return REFCACHE_OK;
+}
+
+// ---------------------------------------------------------------- work lists
+constexpr int kTaskRows = 256;
+
+void add_rows(std::vector<Task>& v, int q0, int qn, int a0, int an, int b0, int bn) {
+  for (int r = 0; r < qn; r += kTaskRows) {
+    Task t{};
+    t.q_row0 = q0 + r;
+    t.q_rows = std::min(kTaskRows, qn - r);
+    t.a_row0 = a0;
+    t.a_len = an;
+    t.b_row0 = b0;
+    t.b_len = bn;
+    v.push_back(t);
+  }
+}
+
+int64_t task_cost(const Task& t) {
+  return static_cast<int64_t>((t.q_rows + 127) / 128) * ((t.a_len + 127) / 128 + (t.b_len + 127) / 128);
+}
+
+// Longest tasks first: the persistent CTAs take items round-robin.
+void order_tasks(std::vector<Task>& v) {
+  std::stable_sort(v.begin(), v.end(), [](const Task& x, const Task& y) { return task_cost(x) > task_cost(y); });
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int check_dims(int batch, int H, int D) {
+  if (batch < 1) return fail(REFCACHE_ERR_INVALID_ARG, "batch must be >= 1 (got %d)", batch);
+  if (H < 1) return fail(REFCACHE_ERR_INVALID_ARG, "num_heads must be >= 1 (got %d)", H);
+  if (D != 64 && D != 128) return fail(REFCACHE_ERR_UNSUPPORTED, "head_dim must be 64 or 128 (got %d)", D);
+  if (static_cast<int64_t>(H) * D > (1 << 20)) return fail(REFCACHE_ERR_INVALID_ARG, "num_heads too large");
+  return REFCACHE_OK;
+}
+
+int check_cu(const int32_t* cu, int batch, const char* name, int64_t max_rows) {
+  if (!cu) return fail(REFCACHE_ERR_INVALID_ARG, "%s is NULL", name);
+  if (cu[0] != 0) return fail(REFCACHE_ERR_INVALID_ARG, "%s[0] must be 0", name);
+  for (int b = 0; b < batch; ++b)
+    if (cu[b + 1] < cu[b]) return fail(REFCACHE_ERR_INVALID_ARG, "%s must be non-decreasing (at %d)", name, b);
+  if (cu[batch] > max_rows) return fail(REFCACHE_ERR_INVALID_ARG, "%s total rows too large", name);
+  return REFCACHE_OK;
+}
+
+int check_scale(float s) {
+  if (!(s > 0.f) || !std::isfinite(s)) return fail(REFCACHE_ERR_INVALID_ARG, "softmax_scale must be finite and > 0");
+  return REFCACHE_OK;
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// ---------------------------------------------------------------- launches
+template <int D>
+int launch_tc(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info, cudaStream_t s) {
+  constexpr uint32_t smem = rc::tc::Smem<D>::kDynamic;
+  const int key = D == 64 ? 0 : 1;
+  if (!info->attr_set[key]) {
+    cudaError_t e = cudaFuncSetAttribute(rc::attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_tc_kernel)");
+    info->attr_set[key] = true;
+  }
+  const int grid = std::min(a.n_items, info->num_sms);
+  rc::attn_tc_kernel<D><<<grid, rc::tc::kThreads, smem, s>>>(maps[0], maps[1], maps[2], maps[3], maps[4], a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "attn_tc_kernel launch");
+  return REFCACHE_OK;
+}
+
+template <int D>
+int launch_mma(const AttnArgs& a, DeviceInfo* info, cudaStream_t s) {
+  constexpr int smem = 5 * 64 * D * 2;
+  const int key = D == 64 ? 2 : 3;
+  if (!info->attr_set[key]) {
+    cudaError_t e = cudaFuncSetAttribute(rc::attn_mma_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_mma_kernel)");
+    info->attr_set[key] = true;
+  }
+  rc::attn_mma_kernel<D><<<a.n_items * 4, 128, smem, s>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "attn_mma_kernel launch");
+  return REFCACHE_OK;
+}
+
+struct Operands {
+  const void* q;
+  int64_t q_rows;
+  const void *ka, *va;
+  int64_t a_rows;
+  const void *kb, *vb;
+  int64_t b_rows;
+  void* o;
+  float* lse;
+};
+
+int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands& op, float scale, DeviceInfo* info,
+                  cudaStream_t s) {
+  if (n_tasks == 0) return REFCACHE_OK;
+  AttnArgs a{};
+  a.tasks = d_tasks;
+  a.n_tasks = n_tasks;
+  a.num_heads = H;
+  a.n_items = n_tasks * H;
+  a.out = static_cast<__nv_bfloat16*>(op.o);
+  a.lse = op.lse;
+  a.row_stride = static_cast<int64_t>(H) * D;
+  a.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634074);
+  a.timeout_ns = g_timeout_ns.load();
+  a.q = static_cast<const __nv_bfloat16*>(op.q);
+  a.ka = static_cast<const __nv_bfloat16*>(op.ka);
+  a.va = static_cast<const __nv_bfloat16*>(op.va);
+  a.kb = static_cast<const __nv_bfloat16*>(op.kb ? op.kb : op.ka);
+  a.vb = static_cast<const __nv_bfloat16*>(op.vb ? op.vb : op.va);
+  if (static_cast<int64_t>(n_tasks) * H > (1ll << 30)) return fail(REFCACHE_ERR_INVALID_ARG, "too many work items");
+  if (g_kernel.load() == REFCACHE_KERNEL_MMA_SYNC)
+    return D == 64 ? launch_mma<64>(a, info, s) : launch_mma<128>(a, info, s);
+  CUtensorMap maps[5];
+  int rc;
+  if ((rc = make_tmap(&maps[0], op.q, op.q_rows, H, D)) != 0) return rc;
+  if ((rc = make_tmap(&maps[1], op.ka, op.a_rows, H, D)) != 0) return rc;
+  if ((rc = make_tmap(&maps[2], op.va, op.a_rows, H, D)) != 0) return rc;
+  if (op.kb && op.b_rows > 0) {
+    if ((rc = make_tmap(&maps[3], op.kb, op.b_rows, H, D)) != 0) return rc;
+    if ((rc = make_tmap(&maps[4], op.vb, op.b_rows, H, D)) != 0) return rc;
+  } else {
+    maps[3] = maps[1];
+    maps[4] = maps[2];
+  }
+  a.dbg_skip_first_load = g_dbg_skip.exchange(0);
+  return D == 64 ? launch_tc<64>(maps, a, info, s) : launch_tc<128>(maps, a, info, s);
+}
+
+struct FullScratch {
+  Task* buf = nullptr;
+  size_t cap = 0;  // tasks
+};
+FullScratch g_full[kMaxDevices];
+std::mutex g_full_mu;
+
+}  // namespace
+
+// ============================================================== the cache handle
+struct refcache {
+  int device = 0;
+  int num_layers = 0, mode = 0, batch = 0, H = 0, D = 0;
+  std::vector<int32_t> cu_live, cu_static, n_anchor;
+  std::vector<int64_t> cache_off;  // [batch+1] cached rows per request, prefix sums
+  int64_t live_rows = 0, static_rows = 0, cache_rows = 0;
+  uint8_t* mem = nullptr;
+  bool owns = false;
+  Task* d_build = nullptr;
+  int n_build = 0;
+  Task* d_step = nullptr;
+  int n_step = 0;
+  CopySeg* d_copy = nullptr;
+  int n_copy = 0;
+  __nv_bfloat16* slots = nullptr;
+  int64_t slot_elems = 0;
+  std::vector<char> built;
+};
+
+namespace {
+
+int cache_plan(int num_layers, int mode, const refcache_segments_t* seg, refcache* h, std::vector<Task>* build_tasks,
+               std::vector<Task>* step_tasks, std::vector<CopySeg>* copies, size_t* total_bytes) {
+  if (!seg) return fail(REFCACHE_ERR_INVALID_ARG, "seg is NULL");
+  if (num_layers < 1) return fail(REFCACHE_ERR_INVALID_ARG, "num_layers must be >= 1");
+  if (mode != REFCACHE_MASK_BEYOND && mode != REFCACHE_MASK_BEYOND_ALT && mode != REFCACHE_MASK_ISOLATED)
+    return fail(REFCACHE_ERR_INVALID_ARG, "unknown mask_mode %d", mode);
+  int rc;
+  if ((rc = check_dims(seg->batch, seg->num_heads, seg->head_dim)) != 0) return rc;
+  const int B = seg->batch;
+  const int64_t max_rows = (1ll << 31) - 1 - 512;
+  if ((rc = check_cu(seg->cu_live, B, "cu_live", max_rows)) != 0) return rc;
+  if ((rc = check_cu(seg->cu_static, B, "cu_static", max_rows)) != 0) return rc;
+  if (!seg->n_anchor) return fail(REFCACHE_ERR_INVALID_ARG, "n_anchor is NULL");
+  std::vector<int64_t> cache_off(B + 1, 0);
+  for (int b = 0; b < B; ++b) {
+    const int ns = seg->cu_static[b + 1] - seg->cu_static[b];
+    const int na = seg->n_anchor[b];
+    if (na < 0 || na > ns) return fail(REFCACHE_ERR_INVALID_ARG, "n_anchor[%d] = %d outside [0, %d]", b, na, ns);
+    if (mode == REFCACHE_MASK_ISOLATED && na != 0)
+      return fail(REFCACHE_ERR_INVALID_ARG, "isolated cache: n_anchor[%d] must be 0", b);
+    if (seg->n_instr) {
+      const int nl = seg->cu_live[b + 1] - seg->cu_live[b];
+      if (seg->n_instr[b] < 0 || seg->n_instr[b] > nl)
+        return fail(REFCACHE_ERR_INVALID_ARG, "n_instr[%d] outside [0, %d]", b, nl);
+    }
+    const int cached = mode == REFCACHE_MASK_BEYOND_ALT ? ns : ns - na;
+    cache_off[b + 1] = cache_off[b] + cached;
+  }
+  if (cache_off[B] > max_rows) return fail(REFCACHE_ERR_INVALID_ARG, "cache rows too large");
+  const int H = seg->num_heads, D = seg->head_dim;
+  std::vector<Task> bt, st;
+  std::vector<CopySeg> cp;
+  for (int b = 0; b < B; ++b) {
+    const int s0 = seg->cu_static[b], ns = seg->cu_static[b + 1] - s0, na = seg->n_anchor[b];
+    const int l0 = seg->cu_live[b], nl = seg->cu_live[b + 1] - l0;
+    const int c0 = static_cast<int>(cache_off[b]), nc = static_cast<int>(cache_off[b + 1] - cache_off[b]);
+    if (mode == REFCACHE_MASK_BEYOND_ALT) {
+      add_rows(bt, s0, na, s0, na, 0, 0);            // anchor rows attend anchors only
+      add_rows(bt, s0 + na, ns - na, s0, ns, 0, 0);  // reference rows attend [ST; R]
+    } else {
+      add_rows(bt, s0, ns, s0, ns, 0, 0);  // [ST; R] rows attend [ST; R] (R only when isolated)
+    }
+    add_rows(st, l0, nl, l0, nl, c0, nc);  // live rows attend their own rows, then the cache
+    if (nc > 0) {
+      CopySeg c{};
+      c.src_row0 = mode == REFCACHE_MASK_BEYOND_ALT ? s0 : s0 + na;
+      c.dst_row0 = c0;
+      c.nrows = nc;
+      cp.push_back(c);
+    }
+  }
+  order_tasks(bt);
+  order_tasks(st);
+  const size_t slot_elems = static_cast<size_t>(cache_off[B]) * H * D;
+  size_t off = 0;
+  off = align_up(off + bt.size() * sizeof(Task), 256);
+  off = align_up(off + st.size() * sizeof(Task), 256);
+  off = align_up(off + cp.size() * sizeof(CopySeg), 256);
+  const size_t total = off + static_cast<size_t>(num_layers) * 2 * slot_elems * sizeof(__nv_bfloat16);
+  if (h) {
+    h->num_layers = num_layers;
+    h->mode = mode;
+    h->batch = B;
+    h->H = H;
+    h->D = D;
+    h->cu_live.assign(seg->cu_live, seg->cu_live + B + 1);
+    h->cu_static.assign(seg->cu_static, seg->cu_static + B + 1);
+    h->n_anchor.assign(seg->n_anchor, seg->n_anchor + B);
+    h->cache_off = cache_off;
+    h->live_rows = seg->cu_live[B];
+    h->static_rows = seg->cu_static[B];
+    h->cache_rows = cache_off[B];
+    h->slot_elems = static_cast<int64_t>(slot_elems);
+    h->n_build = static_cast<int>(bt.size());
+    h->n_step = static_cast<int>(st.size());
+    h->n_copy = static_cast<int>(cp.size());
+  }
+  if (build_tasks) *build_tasks = std::move(bt);
+  if (step_tasks) *step_tasks = std::move(st);
+  if (copies) *copies = std::move(cp);
+  *total_bytes = total;
+  return REFCACHE_OK;
+}
+
+int check_handle_layer(refcache* h, int layer) {
+  if (!h) return fail(REFCACHE_ERR_INVALID_ARG, "cache is NULL");
+  if (layer < 0 || layer >= h->num_layers)
+    return fail(REFCACHE_ERR_INVALID_ARG, "layer %d outside [0, %d)", layer, h->num_layers);
+  return REFCACHE_OK;
+}
+
+int check_ptrs(std::initializer_list<const void*> ps, int64_t rows, const char* what) {
+  if (rows == 0) return REFCACHE_OK;
+  for (const void* p : ps) {
+    if (!p) return fail(REFCACHE_ERR_INVALID_ARG, "%s: NULL tensor pointer", what);
+    if (!aligned16(p)) return fail(REFCACHE_ERR_INVALID_ARG, "%s: tensor pointer not 16-byte aligned", what);
+  }
+  return REFCACHE_OK;
+}
+
+int enter_device(refcache* h, DeviceInfo** info) {
+  int dev = 0;
+  int rc = current_device(&dev, info);
+  if (rc) return rc;
+  if (h && dev != h->device)
+    return fail(REFCACHE_ERR_INVALID_ARG, "current device %d is not the cache's device %d", dev, h->device);
+  return REFCACHE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t refcache_bytes(int num_layers, int mask_mode, const refcache_segments_t* seg) {
+  size_t total = 0;
+  if (cache_plan(num_layers, mask_mode, seg, nullptr, nullptr, nullptr, nullptr, &total) != 0) return 0;
+  return total;
+}
+
+int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refcache_segments_t* seg, void* dev_mem,
+                    size_t dev_bytes) {
+  if (!out) return fail(REFCACHE_ERR_INVALID_ARG, "out is NULL");
+  refcache* h = new refcache();
+  std::vector<Task> bt, st;
+  std::vector<CopySeg> cp;
+  size_t total = 0;
+  int rc = cache_plan(num_layers, mask_mode, seg, h, &bt, &st, &cp, &total);
+  if (rc) {
+    delete h;
+    return rc;
+  }
+  if (dev_mem) {
+    if (dev_bytes < total) {
+      delete h;
+      return fail(REFCACHE_ERR_OOM, "given %zu bytes, need %zu", dev_bytes, total);
+    }
+    if (reinterpret_cast<uintptr_t>(dev_mem) & 255u) {
+      delete h;
+      return fail(REFCACHE_ERR_INVALID_ARG, "dev_mem must be 256-byte aligned");
+    }
+  }
+  DeviceInfo* info = nullptr;
+  if ((rc = current_device(&h->device, &info)) != 0) {
+    delete h;
+    return rc;
+  }
+  if (dev_mem) {
+    h->mem = static_cast<uint8_t*>(dev_mem);
+  } else {
+    cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&h->mem), total);
+    if (e != cudaSuccess) {
+      delete h;
+      return fail(REFCACHE_ERR_OOM, "cudaMalloc(%zu): %s", total, cudaGetErrorString(e));
+    }
+    h->owns = true;
+  }
+  size_t off = 0;
+  h->d_build = reinterpret_cast<Task*>(h->mem + off);
+  off = align_up(off + bt.size() * sizeof(Task), 256);
+  h->d_step = reinterpret_cast<Task*>(h->mem + off);
+  off = align_up(off + st.size() * sizeof(Task), 256);
+  h->d_copy = reinterpret_cast<CopySeg*>(h->mem + off);
+  off = align_up(off + cp.size() * sizeof(CopySeg), 256);
+  h->slots = reinterpret_cast<__nv_bfloat16*>(h->mem + off);
+  cudaError_t e = cudaSuccess;
+  if (!bt.empty() && e == cudaSuccess) e = cudaMemcpy(h->d_build, bt.data(), bt.size() * sizeof(Task), cudaMemcpyHostToDevice);
+  if (!st.empty() && e == cudaSuccess) e = cudaMemcpy(h->d_step, st.data(), st.size() * sizeof(Task), cudaMemcpyHostToDevice);
+  if (!cp.empty() && e == cudaSuccess) e = cudaMemcpy(h->d_copy, cp.data(), cp.size() * sizeof(CopySeg), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) {
+    if (h->owns) cudaFree(h->mem);
+    delete h;
+    return cuda_fail(e, "cudaMemcpy(work tables)");
+  }
+  h->built.assign(num_layers, 0);
+  *out = h;
+  return REFCACHE_OK;
+}
+
+void refcache_destroy(refcache_t* h) {
+  if (!h) return;
+  if (h->owns && h->mem) {
+    int prev = 0;
+    cudaGetDevice(&prev);
+    cudaSetDevice(h->device);
+    cudaDeviceSynchronize();
+    cudaFree(h->mem);
+    cudaSetDevice(prev);
+  }
+  delete h;
+}
+
+int refcache_kv_ptr(refcache_t* h, int layer, void** k_slot, void** v_slot, int64_t* rows) {
+  int rc = check_handle_layer(h, layer);
+  if (rc) return rc;
+  __nv_bfloat16* k = h->slots + static_cast<int64_t>(layer) * 2 * h->slot_elems;
+  if (k_slot) *k_slot = k;
+  if (v_slot) *v_slot = k + h->slot_elems;
+  if (rows) *rows = h->cache_rows;
+  return REFCACHE_OK;
+}
+
+int refcache_layer_built(refcache_t* h, int layer) {
+  int rc = check_handle_layer(h, layer);
+  if (rc) return rc;
+  return h->built[layer] ? 1 : 0;
+}
+
+int refcache_build(refcache_t* h, int layer, const void* q_static, const void* k_static, const void* v_static,
+                   void* o_static, float* lse_static, float softmax_scale, void* stream) {
+  int rc = check_handle_layer(h, layer);
+  if (rc) return rc;
+  if ((rc = check_scale(softmax_scale)) != 0) return rc;
+  if ((rc = check_ptrs({q_static, k_static, v_static, o_static}, h->static_rows, "refcache_build")) != 0) return rc;
+  DeviceInfo* info = nullptr;
+  if ((rc = enter_device(h, &info)) != 0) return rc;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  void *kslot = nullptr, *vslot = nullptr;
+  refcache_kv_ptr(h, layer, &kslot, &vslot, nullptr);
+  if (h->n_copy > 0) {
+    const int row_u4 = h->H * h->D * 2 / 16;
+    dim3 grid(static_cast<unsigned>(std::min<int64_t>(1024, (h->cache_rows * row_u4 + 255) / 256 / h->n_copy + 1)),
+              static_cast<unsigned>(h->n_copy));
+    rc::copy_rows_kernel<<<grid, 256, 0, s>>>(h->d_copy, static_cast<const uint4*>(k_static),
+                                              static_cast<const uint4*>(v_static), static_cast<uint4*>(kslot),
+                                              static_cast<uint4*>(vslot), row_u4);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "copy_rows_kernel launch");
+  }
+  Operands op{q_static, h->static_rows, k_static, v_static, h->static_rows, nullptr, nullptr, 0, o_static, lse_static};
+  rc = run_attention(h->d_build, h->n_build, h->H, h->D, op, softmax_scale, info, s);
+  if (rc) return rc;
+  h->built[layer] = 1;
+  return REFCACHE_OK;
+}
+
+int step_attention(refcache_t* h, int layer, const void* q_live, const void* k_live, const void* v_live, void* o_live,
+                   float* lse_live, float softmax_scale, void* stream) {
+  int rc = check_handle_layer(h, layer);
+  if (rc) return rc;
+  if (!h->built[layer]) return fail(REFCACHE_ERR_NOT_BUILT, "layer %d has not been built", layer);
+  if ((rc = check_scale(softmax_scale)) != 0) return rc;
+  if ((rc = check_ptrs({q_live, k_live, v_live, o_live}, h->live_rows, "step_attention")) != 0) return rc;
+  DeviceInfo* info = nullptr;
+  if ((rc = enter_device(h, &info)) != 0) return rc;
+  void *kslot = nullptr, *vslot = nullptr;
+  refcache_kv_ptr(h, layer, &kslot, &vslot, nullptr);
+  Operands op{q_live, h->live_rows, k_live, v_live, h->live_rows, kslot, vslot, h->cache_rows, o_live, lse_live};
+  return run_attention(h->d_step, h->n_step, h->H, h->D, op, softmax_scale, info, static_cast<cudaStream_t>(stream));
+}
+
+int full_attention(int batch, int num_heads, int head_dim, const int32_t* cu_seqlens, const void* q, const void* k,
+                   const void* v, void* o, float* lse, float softmax_scale, void* stream) {
+  int rc = check_dims(batch, num_heads, head_dim);
+  if (rc) return rc;
+  if ((rc = check_cu(cu_seqlens, batch, "cu_seqlens", (1ll << 31) - 1 - 512)) != 0) return rc;
+  if ((rc = check_scale(softmax_scale)) != 0) return rc;
+  const int64_t rows = cu_seqlens[batch];
+  if ((rc = check_ptrs({q, k, v, o}, rows, "full_attention")) != 0) return rc;
+  DeviceInfo* info = nullptr;
+  if ((rc = enter_device(nullptr, &info)) != 0) return rc;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  std::vector<Task> tasks;
+  for (int b = 0; b < batch; ++b) {
+    const int s0 = cu_seqlens[b], n = cu_seqlens[b + 1] - s0;
+    add_rows(tasks, s0, n, s0, n, 0, 0);
+  }
+  order_tasks(tasks);
+  if (tasks.empty()) return REFCACHE_OK;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  Task* d_tasks = nullptr;
+  {
+    std::lock_guard<std::mutex> lk(g_full_mu);
+    FullScratch& fs = g_full[dev];
+    if (fs.cap < tasks.size()) {
+      if (fs.buf) {
+        cudaError_t e = cudaStreamSynchronize(s);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+        cudaFree(fs.buf);
+        fs.buf = nullptr;
+        fs.cap = 0;
+      }
+      const size_t cap = std::max<size_t>(tasks.size(), 1024);
+      cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&fs.buf), cap * sizeof(Task));
+      if (e != cudaSuccess) return fail(REFCACHE_ERR_OOM, "cudaMalloc(work list): %s", cudaGetErrorString(e));
+      fs.cap = cap;
+    }
+    d_tasks = fs.buf;
+    cudaError_t e = cudaMemcpyAsync(d_tasks, tasks.data(), tasks.size() * sizeof(Task), cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync(work list)");
+  }
+  Operands op{q, rows, k, v, rows, nullptr, nullptr, 0, o, lse};
+  return run_attention(d_tasks, static_cast<int>(tasks.size()), num_heads, head_dim, op, softmax_scale, info, s);
+}
+
+int refcache_status(void* stream) {
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+  int v = 0;
+  e = cudaMemcpyFromSymbol(&v, rc::g_rc_status, sizeof(int));
+  if (e != cudaSuccess) return cuda_fail(e, "read device error word");
+  if (v != 0) {
+    const int zero = 0;
+    e = cudaMemcpyToSymbol(rc::g_rc_status, &zero, sizeof(int));
+    if (e != cudaSuccess) return cuda_fail(e, "clear device error word");
+    return fail(REFCACHE_ERR_TIMEOUT, "a kernel wait ran out (site %d)", v - RC_DEV_TIMEOUT_BASE);
+  }
+  return REFCACHE_OK;
+}
+
+uint64_t refcache_set_wait_timeout_ns(uint64_t ns) { return g_timeout_ns.exchange(ns ? ns : 1); }
+
+int refcache_set_kernel(int kernel) {
+  if (kernel != REFCACHE_KERNEL_TCGEN05 && kernel != REFCACHE_KERNEL_MMA_SYNC)
+    return fail(REFCACHE_ERR_INVALID_ARG, "unknown kernel %d", kernel);
+  return g_kernel.exchange(kernel);
+}
+
+void refcache_debug_skip_first_load(int on) { g_dbg_skip.store(on ? 1 : 0); }
+
+int refcache_last_error(char* buf, size_t n) {
+  if (buf && n > 0) {
+    std::strncpy(buf, g_last_error.c_str(), n - 1);
+    buf[n - 1] = '\0';
+  }
+  return static_cast<int>(g_last_error.size());
+}
+
+const char* refcache_version(void) { return "refcache 0.1.0 (sm_103a)"; }
+
+}  // extern "C"

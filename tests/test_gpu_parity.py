@@ -1,0 +1,206 @@
+"""CUDA path (through the C ABI) against the CPU oracle on the same seeded inputs.
+
+Bar: max |gpu - oracle| <= 2e-2 and mean |gpu - oracle| <= 2e-3 for outputs,
+|lse| error <= 2e-3; cached K/V and the exact-caching invariant bit for bit.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads
+from paper_2608_21229_gb300 import refcache as rcb
+
+import parity_utils as pu
+
+pytestmark = pytest.mark.gpu
+
+KERNELS = ["tcgen05", "mma_sync"]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.fail("GPU tests need a CUDA device")
+    rcb.load()
+    oracle.build()
+    yield
+    rcb.set_kernel("tcgen05")
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("mode", ["beyond", "beyond_alt"])
+def test_tiny_full_compare(kernel, mode):
+    run = pu.GpuRun(workloads.TINY, mode=mode, kernel=kernel)
+    pu.full_compare(run)
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_tiny_isolated_full_compare(kernel):
+    w = workloads.Workload("tiny_isolated", 4, 64, (workloads.Request(0, 64, 256, 256),), 0)
+    run = pu.GpuRun(w, mode="isolated", kernel=kernel)
+    pu.full_compare(run)
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_edit512_2ref_full_compare(kernel):
+    run = pu.GpuRun(workloads.EDIT_512_2REF, kernel=kernel)
+    pu.full_compare(run)
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("mode", ["beyond", "beyond_alt", "isolated"])
+@pytest.mark.parametrize("head_dim", [64, 128])
+@pytest.mark.parametrize("seed", [11, 12])
+def test_ragged_small_full_compare(kernel, mode, head_dim, seed):
+    """Several requests with ragged lengths (0, 1, odd, across tile edges)."""
+    rng = np.random.default_rng(seed)
+    reqs = list(workloads.random_requests(rng, 3, max_len=300))
+    reqs.append(workloads.Request(1, 0, 1, 1))
+    reqs.append(workloads.Request(0, 0, 0, 5))
+    reqs.append(workloads.Request(3, 2, 0, 0))
+    if mode == "isolated":
+        reqs = [workloads.Request(0, r.n_lt, r.n_x, r.n_r) for r in reqs]
+    w = workloads.Workload(f"ragged_small_{seed}", 3, head_dim, tuple(reqs), seed)
+    run = pu.GpuRun(w, mode=mode, kernel=kernel)
+    pu.full_compare(run)
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_edit1024_5ref_sampled(kernel):
+    run = pu.GpuRun(workloads.EDIT_1024_5REF, kernel=kernel)
+    pu.sampled_compare(run, seed=5)
+
+
+@pytest.mark.parametrize("refs", [1, 10])
+def test_sweep_sampled(refs):
+    w = [x for x in workloads.SWEEP_1024 if x.requests[0].n_r == refs * 4096][0]
+    run = pu.GpuRun(w, kernel="tcgen05")
+    pu.sampled_compare(run, seed=refs, per_request=16)
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("mode", ["beyond", "beyond_alt"])
+def test_ragged_serving_batch_sampled(kernel, mode):
+    run = pu.GpuRun(workloads.RAGGED_4REQ, mode=mode, kernel=kernel)
+    pu.sampled_compare(run, seed=7, per_request=16)
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_exact_caching_invariant_bitwise(kernel):
+    """Sec. 3.1 / 3.3: the prefill outputs and the cache bytes do not depend
+    on the live inputs; rebuilding after steps with other live data, and on a
+    second layer, reproduces them bit for bit."""
+    w = workloads.EDIT_512_2REF
+    rcb.set_kernel(kernel)
+    seg = rcb.Segments.from_workload(w)
+    H, D = w.num_heads, w.head_dim
+    cache = rcb.RefCache(seg, num_layers=2)
+    qs, ks, vs = (t.cuda() for t in workloads.static_qkv(w))
+    o1 = torch.empty(seg.static_rows, H, D, dtype=torch.bfloat16, device="cuda")
+    o2 = torch.empty_like(o1)
+    cache.build(0, qs, ks, vs, o1)
+    k0, v0 = (t.clone() for t in cache.kv(0))
+    ol = torch.empty(seg.live_rows, H, D, dtype=torch.bfloat16, device="cuda")
+    for step in range(3):
+        ql, kl, vl = (t.cuda() for t in workloads.live_qkv(w, step=step))
+        cache.step(0, ql, kl, vl, ol)
+    cache.build(1, qs, ks, vs, o2)
+    o3 = torch.empty_like(o1)
+    cache.build(0, qs, ks, vs, o3)
+    torch.cuda.synchronize()
+    assert rcb.status() == rcb.OK
+    assert torch.equal(o1.view(torch.int16), o2.view(torch.int16))
+    assert torch.equal(o1.view(torch.int16), o3.view(torch.int16))
+    for layer in (0, 1):
+        k, v = cache.kv(layer)
+        assert torch.equal(k.view(torch.int16), k0.view(torch.int16))
+        assert torch.equal(v.view(torch.int16), v0.view(torch.int16))
+    # the cache holds exactly the R rows' K and V given (Eq. 2)
+    r = w.requests[0]
+    assert torch.equal(k0.view(torch.int16), ks[r.n_st:].view(torch.int16))
+    assert torch.equal(v0.view(torch.int16), vs[r.n_st:].view(torch.int16))
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_step_depends_on_cache_not_on_static_inputs(kernel):
+    """The step reads K/V of R only from the cache: overwriting the prefill
+    input tensors after the build leaves the step output unchanged."""
+    w = workloads.TINY
+    rcb.set_kernel(kernel)
+    seg = rcb.Segments.from_workload(w)
+    H, D = w.num_heads, w.head_dim
+    cache = rcb.RefCache(seg)
+    qs, ks, vs = (t.cuda() for t in workloads.static_qkv(w))
+    os_ = torch.empty(seg.static_rows, H, D, dtype=torch.bfloat16, device="cuda")
+    cache.build(0, qs, ks, vs, os_)
+    ql, kl, vl = (t.cuda() for t in workloads.live_qkv(w))
+    a = torch.empty(seg.live_rows, H, D, dtype=torch.bfloat16, device="cuda")
+    b = torch.empty_like(a)
+    cache.step(0, ql, kl, vl, a)
+    ks.normal_()
+    vs.normal_()
+    cache.step(0, ql, kl, vl, b)
+    torch.cuda.synchronize()
+    assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("w", [workloads.TINY, workloads.EDIT_512_2REF], ids=lambda w: w.name)
+def test_full_attention_matches_oracle(kernel, w):
+    """The full-recompute baseline: every row of [LT; X; R] sees every key (Sec. 3.2)."""
+    rcb.set_kernel(kernel)
+    r = w.requests[0]
+    n = r.n_lt + r.n_x + r.n_r
+    H, D = w.num_heads, w.head_dim
+    q, k, v = (workloads.randn_bf16((n, H, D), w.seed, f"full_{t}") for t in "qkv")
+    o = torch.empty(n, H, D, dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty(n, H, dtype=torch.float32, device="cuda")
+    rcb.full_attention([0, n], q.cuda(), k.cuda(), v.cuda(), o, lse)
+    torch.cuda.synchronize()
+    assert rcb.status() == rcb.OK
+    rng = np.random.default_rng(3)
+    rows = pu.sample_rows(n, rng, 64)
+    pairs = np.stack([rows, rng.integers(0, H, rows.size)], 1).astype(np.int32)
+    ref_o, ref_l = oracle.full(pu.bits(q), pu.bits(k), pu.bits(v), 1 / math.sqrt(D), pairs)
+    go = pu.f64(o)[pairs[:, 0], pairs[:, 1]]
+    gl = pu.f64(lse)[pairs[:, 0], pairs[:, 1]]
+    pu.check_close(go, ref_o, gl, ref_l, "full")
+
+
+def test_kernels_agree_closely():
+    """The two kernels compute the same function (different rounding order)."""
+    w = workloads.EDIT_512_2REF
+    a = pu.GpuRun(w, kernel="tcgen05")
+    b = pu.GpuRun(w, kernel="mma_sync", static=a.static, live=a.live)
+    d = (pu.f64(a.o_live) - pu.f64(b.o_live))
+    assert np.abs(d).max() < 2e-2 and np.abs(d).mean() < 1e-3
+
+
+def test_not_built_and_bad_args_are_rejected():
+    w = workloads.TINY
+    seg = rcb.Segments.from_workload(w)
+    cache = rcb.RefCache(seg, num_layers=2)
+    H, D = w.num_heads, w.head_dim
+    ql, kl, vl = (t.cuda() for t in workloads.live_qkv(w))
+    o = torch.empty(seg.live_rows, H, D, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(rcb.RefCacheError) as e:
+        cache.step(1, ql, kl, vl, o)
+    assert e.value.code == rcb.ERR_NOT_BUILT
+    qs, ks, vs = (t.cuda() for t in workloads.static_qkv(w))
+    os_ = torch.empty(seg.static_rows, H, D, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(rcb.RefCacheError) as e:
+        cache.build(0, qs, ks, vs, os_, scale=-1.0)
+    assert e.value.code == rcb.ERR_INVALID_ARG
+    with pytest.raises(rcb.RefCacheError) as e:
+        cache.build(5, qs, ks, vs, os_)
+    assert e.value.code == rcb.ERR_INVALID_ARG
+    # misaligned base pointer (2-byte offset view)
+    flat = torch.empty(seg.static_rows * H * D + 8, dtype=torch.bfloat16, device="cuda")
+    mis = flat[1:1 + seg.static_rows * H * D].view(seg.static_rows, H, D)
+    with pytest.raises(rcb.RefCacheError) as e:
+        cache.build(0, mis, ks, vs, os_)
+    assert e.value.code == rcb.ERR_INVALID_ARG
+    assert rcb.status() == rcb.OK

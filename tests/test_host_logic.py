@@ -1,0 +1,45 @@
+"""Host logic: the accounting the benchmark reports against the App. C model,
+and the seeded input generators."""
+import pytest
+import torch
+
+import workloads
+from oracle import cost_model as cm
+from paper_2608_21229_gb300 import accounting as acc
+
+
+@pytest.mark.parametrize("w", [workloads.TINY, workloads.EDIT_512_2REF, workloads.EDIT_1024_5REF]
+                         + list(workloads.SWEEP_1024), ids=lambda w: w.name)
+def test_accounting_equals_app_c_model(w):
+    r = w.requests[0]
+    s = r.n_lt + r.n_x
+    assert acc.prefill_units(w.requests) == cm.c_pre(r.n_r, r.n_st)
+    assert acc.step_units(w.requests) == cm.c_step(r.n_r, s)
+    assert 40 * acc.full_units(w.requests) == cm.c_full(r.n_r, s, 40)
+    assert acc.modelled_ratio(w.requests, 40) == pytest.approx(cm.speedup(r.n_r, r.n_st, s, 40), rel=1e-12)
+    assert acc.flops(1, 24, 128) == cm.flops_per_unit(128) * 24
+    assert acc.prefill_units(w.requests) - acc.prefill_units(
+        [workloads.Request(0, r.n_lt, r.n_x, r.n_r)]) == cm.anchor_overhead(r.n_r, r.n_st)
+
+
+def test_headline_step_flops():
+    w = workloads.EDIT_1024_5REF
+    f = acc.flops(acc.step_units(w.requests), w.num_heads, w.head_dim)
+    assert f == 4 * 128 * 24 * 4608 * (4608 + 20480)
+    assert acc.cache_bytes(w.requests, 24, 128) == 2 * 20480 * 24 * 128 * 2
+
+
+def test_generators_are_deterministic_and_distinct():
+    a = workloads.randn_bf16((64, 2, 8), 0, "x")
+    b = workloads.randn_bf16((64, 2, 8), 0, "x")
+    c = workloads.randn_bf16((64, 2, 8), 0, "y")
+    assert a.dtype == torch.bfloat16 and torch.equal(a, b) and not torch.equal(a, c)
+    assert abs(float(workloads.randn_bf16((4096, 64), 1, "z").float().std()) - 1.0) < 0.02
+
+
+def test_workload_shapes():
+    w = workloads.RAGGED_4REQ
+    assert w.batch == 4 and [r.n_r // 1024 if r.n_x == 1024 else r.n_r // 4096 for r in w.requests] == [1, 3, 5, 8]
+    assert w.cu_live[-1] == sum(r.n_lt + r.n_x for r in w.requests)
+    q, k, v = workloads.static_qkv(workloads.TINY)
+    assert q.shape == (288, 4, 64)
