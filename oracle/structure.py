@@ -2,13 +2,13 @@
 
 A layer-shared block mask M over a block set V; ``attends(q, k)`` says that
 block q attends to block k (the paper writes M[k, q] = 1 for the same
-relation, Eq. 7).  Unrolling across depth gives nodes (b, l) for l = 0..L,
+relation, App. A Eq. blockrec).  Unrolling across depth gives nodes (b, l) for l = 0..L,
 residual edges (b, l-1) -> (b, l) and attention edges (k, l-1) -> (q, l)
 whenever q attends k.
 
-  StructCacheable(R)    <=>  (X, 0) reaches no (R, l), l = 1..L      (Eq. 8)
+  StructCacheable(R)    <=>  (X, 0) reaches no (R, l), l = 1..L  (Eq. def-cache)
   LiveTextReachable(R)  <=>  (LT, l) reaches (R, m) for some 1 <= l < m <= L
-                                                                      (Eq. 9)
+                                                        (Eq. def-instr)
 Theorem 1: with L >= 2, a layer-shared mask on {LT, X, R} and LT attending X,
 no mask satisfies both.
 """
