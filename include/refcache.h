@@ -175,6 +175,33 @@ REFCACHE_API int full_attention(int batch, int num_heads, int head_dim, const in
                    void* stream);
 
 /*
+ * full_attention for callers that cannot allocate device memory -- e.g. code
+ * running under a custom or pooled allocator that forbids cudaMalloc, or a
+ * host runtime that must not grow GPU memory after start-up.  The paper has
+ * no counterpart; this is a deployment variant of full_attention above.
+ *
+ * Same arguments, semantics and results as full_attention, but the work list
+ * lives in a fixed array in the library's static device memory (held by every
+ * GPU that loads the library until the process exits), so the call allocates
+ * nothing: no cudaMalloc, no cudaFree, no allocating library routine.  The
+ * caller still passes (and owns) q, k, v, o and lse.
+ *   - The array holds REFCACHE_NOALLOC_MAX_TASKS work items; a request of n
+ *     rows needs ceil(n / 256) of them.  Larger inputs are rejected with
+ *     REFCACHE_ERR_INVALID_ARG and a message naming the limit.
+ *   - The first call on each device looks up the array's device address with
+ *     that device current (a one-time set-up); make that first call before any
+ *     stream capture.
+ *   - Every call rewrites the whole work list it uses, so no state carries
+ *     over, but all calls share the one array: calls whose kernels overlap on
+ *     the GPU (different streams, or other threads) race.  Order them on one
+ *     stream.
+ */
+#define REFCACHE_NOALLOC_MAX_TASKS 16384
+REFCACHE_API int full_attention_noalloc(int batch, int num_heads, int head_dim, const int32_t* cu_seqlens,
+                                        const void* q, const void* k, const void* v, void* o, float* lse,
+                                        float softmax_scale, void* stream);
+
+/*
  * Synchronise `stream`, then read and clear the current device's error word
  * written by kernels whose bounded waits ran out.  Returns REFCACHE_OK,
  * REFCACHE_ERR_TIMEOUT or REFCACHE_ERR_CUDA.

@@ -249,6 +249,13 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
   return D == 64 ? launch_tc<64>(maps, a, info, s) : launch_tc<128>(maps, a, info, s);
 }
 
+// Work list of full_attention_noalloc: a fixed array in static device memory
+// (no allocation at call time), shared by every call on a device.
+__device__ __align__(256) static Task g_noalloc_tasks[REFCACHE_NOALLOC_MAX_TASKS];
+Task* g_noalloc_dev_ptr[kMaxDevices];
+std::mutex g_noalloc_mu;
+Task g_noalloc_host[REFCACHE_NOALLOC_MAX_TASKS];  // host staging, guarded by g_noalloc_mu
+
 struct FullScratch {
   Task* buf = nullptr;
   size_t cap = 0;  // tasks
@@ -573,6 +580,62 @@ int full_attention(int batch, int num_heads, int head_dim, const int32_t* cu_seq
   }
   Operands op{q, rows, k, v, rows, nullptr, nullptr, 0, o, lse};
   return run_attention(d_tasks, static_cast<int>(tasks.size()), num_heads, head_dim, op, softmax_scale, info, s);
+}
+
+int full_attention_noalloc(int batch, int num_heads, int head_dim, const int32_t* cu_seqlens, const void* q,
+                           const void* k, const void* v, void* o, float* lse, float softmax_scale, void* stream) {
+  int rc = check_dims(batch, num_heads, head_dim);
+  if (rc) return rc;
+  if ((rc = check_cu(cu_seqlens, batch, "cu_seqlens", (1ll << 31) - 1 - 512)) != 0) return rc;
+  if ((rc = check_scale(softmax_scale)) != 0) return rc;
+  int64_t n_tasks = 0;
+  for (int b = 0; b < batch; ++b) n_tasks += (cu_seqlens[b + 1] - cu_seqlens[b] + kTaskRows - 1) / kTaskRows;
+  if (n_tasks > REFCACHE_NOALLOC_MAX_TASKS)
+    return fail(REFCACHE_ERR_INVALID_ARG,
+                "full_attention_noalloc: %lld work items exceed the static limit of %d (256 query rows each)",
+                static_cast<long long>(n_tasks), REFCACHE_NOALLOC_MAX_TASKS);
+  const int64_t rows = cu_seqlens[batch];
+  if ((rc = check_ptrs({q, k, v, o}, rows, "full_attention_noalloc")) != 0) return rc;
+  DeviceInfo* info = nullptr;
+  if ((rc = enter_device(nullptr, &info)) != 0) return rc;
+  if (n_tasks == 0) return REFCACHE_OK;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  std::lock_guard<std::mutex> lk(g_noalloc_mu);
+  if (!g_noalloc_dev_ptr[dev]) {
+    // one-time set-up per device, with that device current: the host-side name
+    // of a __device__ array is not a device address, so look the address up
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_tasks);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(work list)");
+    g_noalloc_dev_ptr[dev] = static_cast<Task*>(p);
+  }
+  int n = 0;
+  for (int b = 0; b < batch; ++b) {
+    const int s0 = cu_seqlens[b], len = cu_seqlens[b + 1] - s0;
+    for (int r = 0; r < len; r += kTaskRows) {
+      Task t{};
+      t.q_row0 = s0 + r;
+      t.q_rows = std::min(kTaskRows, len - r);
+      t.a_row0 = s0;
+      t.a_len = len;
+      g_noalloc_host[n++] = t;
+    }
+  }
+  // the same longest-first order as full_attention (ties by row, so the order is total)
+  std::sort(g_noalloc_host, g_noalloc_host + n, [](const Task& x, const Task& y) {
+    const int64_t cx = task_cost(x), cy = task_cost(y);
+    return cx != cy ? cx > cy : x.q_row0 < y.q_row0;
+  });
+  // pageable source: the copy is staged before cudaMemcpyAsync returns, so the
+  // host array may be reused by the next call
+  e = cudaMemcpyAsync(g_noalloc_dev_ptr[dev], g_noalloc_host, static_cast<size_t>(n) * sizeof(Task),
+                      cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync(work list)");
+  Operands op{q, rows, k, v, rows, nullptr, nullptr, 0, o, lse};
+  return run_attention(g_noalloc_dev_ptr[dev], n, num_heads, head_dim, op, softmax_scale, info, s);
 }
 
 int refcache_status(void* stream) {

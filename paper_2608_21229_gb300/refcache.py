@@ -29,7 +29,9 @@ EXPORTED = (
     "refcache_bytes", "refcache_create", "refcache_destroy", "refcache_kv_ptr", "refcache_layer_built",
     "refcache_build", "step_attention", "full_attention", "refcache_status", "refcache_set_wait_timeout_ns",
     "refcache_set_kernel", "refcache_debug_skip_first_load", "refcache_last_error", "refcache_version",
+    "full_attention_noalloc",
 )
+NOALLOC_MAX_TASKS = 16384
 
 
 class RefCacheError(RuntimeError):
@@ -75,6 +77,8 @@ def load(path: Optional[str] = None):
     L.refcache_build.argtypes = [vp, i32, vp, vp, vp, vp, vp, f32, vp]
     L.step_attention.argtypes = [vp, i32, vp, vp, vp, vp, vp, f32, vp]
     L.full_attention.argtypes = [i32, i32, i32, ctypes.POINTER(ctypes.c_int32), vp, vp, vp, vp, vp, f32, vp]
+    L.full_attention_noalloc.argtypes = [i32, i32, i32, ctypes.POINTER(ctypes.c_int32), vp, vp, vp, vp, vp, f32,
+                                         vp]
     L.refcache_status.argtypes = [vp]
     L.refcache_set_wait_timeout_ns.argtypes = [ctypes.c_uint64]
     L.refcache_set_wait_timeout_ns.restype = ctypes.c_uint64
@@ -267,3 +271,15 @@ def full_attention(cu_seqlens, q, k, v, o, lse=None, scale=None, stream=None):
     scale = default_scale(D) if scale is None else scale
     _check(load().full_attention(len(cu) - 1, H, D, _arr(cu), _ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse),
                                  scale, _stream(stream)))
+
+
+def full_attention_noalloc(cu_seqlens, q, k, v, o, lse=None, scale=None, stream=None):
+    """full_attention whose work list sits in the library's static device
+    memory: the call allocates no device memory (see include/refcache.h)."""
+    rows, H, D = q.shape
+    cu = list(cu_seqlens)
+    for name, t in (("q", q), ("k", k), ("v", v), ("o", o)):
+        _check_thd(name, t, cu[-1], H, D)
+    scale = default_scale(D) if scale is None else scale
+    _check(load().full_attention_noalloc(len(cu) - 1, H, D, _arr(cu), _ptr(q), _ptr(k), _ptr(v), _ptr(o),
+                                         _ptr(lse), scale, _stream(stream)))
