@@ -186,7 +186,7 @@ REFCACHE_API int full_attention(int batch, int num_heads, int head_dim, const in
  * nothing: no cudaMalloc, no cudaFree, no allocating library routine.  The
  * caller still passes (and owns) q, k, v, o and lse.
  *   - The array holds REFCACHE_NOALLOC_MAX_TASKS work items; a request of n
- *     rows needs ceil(n / 256) of them.  Larger inputs are rejected with
+ *     rows needs ceil(n / 128) of them.  Larger inputs are rejected with
  *     REFCACHE_ERR_INVALID_ARG and a message naming the limit.
  *   - The first call on each device looks up the array's device address with
  *     that device current (a one-time set-up); make that first call before any

@@ -6,26 +6,36 @@
 // scores, softmax and accumulation in fp32 and P rounded to bf16 for P.V.
 //
 // CTA organisation (one persistent CTA per SM, 320 threads):
-//   warps 0-3  softmax group 0: query tile 0 (item rows 0..127), one row per thread
-//   warps 4-7  softmax group 1: query tile 1 (item rows 128..255)
-//   warp 8     TMA producer: Q tiles once per item, then K_j and V_j tiles
-//              of 128 keys into a ring of NS shared-memory slots
-//   warp 9     MMA issuer (one thread): S_i = Q_i K_j^T, O_i += P_i V_j;
-//              also allocates and frees tensor memory
-// Tensor memory (512 columns x 128 lanes of 32 bit):
-//   S_0 cols [0,128)   S_1 cols [128,256)   O_0 cols [256,256+D)   O_1 [384,384+D)
-//   P_i (bf16, two per column) overwrites the first 64 columns of S_i once
-//   the softmax has read S_i; the P.V MMA reads P_i straight from TMEM.
-// Per key tile j the MMA thread issues S_0, S_1, then (after each softmax
-// group has written P_i) O_0 += P_0 V_j and O_1 += P_1 V_j, so the softmax of
-// one query tile overlaps the tensor-core work of the other.
-// Rescaling of O is lazy: a row's running maximum is only moved (and its O
-// row in TMEM multiplied down) when a new score exceeds it by more than 2^8.
+//   warps 0-7  softmax: row r of the item's 128-row query tile is shared by
+//              thread r of warps 0-3 (score columns 0-63) and thread r of
+//              warps 4-7 (columns 64-127); the two exchange their partial
+//              row maxima through shared memory once per tile
+//   warp 8     TMA producer: the item's Q tile, then K and V tiles of 128
+//              keys into a ring of kNumSlots shared-memory slots
+//   warp 9     MMA issuer (one thread); also allocates and frees TMEM
 //
-// Shared memory: Q_0, Q_1 and NS ring slots of 128 rows x D bf16 each, every
-// tile stored as D/64 TMA boxes of 128 rows x 128 bytes with the 128-byte
-// swizzle (the canonical K-major layout for Q and K; V is read as the
-// MN-major B operand of P.V from the same layout).
+// The key tiles of all items a CTA runs form one stream t = 0, 1, 2, ...
+// For tile t the MMA thread computes S_t = Q K_t^T and O += P_t V_t.  The
+// MMAs are issued in pairs: pair t interleaves, instruction by instruction,
+// the 8 MMAs of O += P_t V_t with the MMAs of S_{t+2} = Q K_{t+2}^T (the
+// latter may belong to the next item).  The tensor core then runs a stream
+// that alternates the two instruction kinds at every MMA, which keeps it at
+// full rate, whereas long runs of one kind followed by the other drain its
+// pipeline at every switch.  While pair t runs, the softmax turns S_{t+1}
+// into P_{t+1}, so the softmax of one tile overlaps the MMAs of the others.
+//
+// Tensor memory (512 columns x 128 lanes of 32 bit):
+//   S buffers  [0,128) [128,256)   tile t uses buffer t % 2 (fp32 scores)
+//   P buffers  [256,320) [320,384) tile t uses buffer t % 2 (bf16 pairs,
+//              read by the P.V MMA as its A operand)
+//   O          [384, 384 + D)      fp32 accumulator of the current item
+// Rescaling of O is lazy: a row's running maximum is only moved (and its O
+// row multiplied down) when a new score exceeds it by more than 2^8.
+//
+// Shared memory: two Q tile buffers (item i uses buffer i % 2) and a ring of
+// kNumSlots tiles of 128 rows x D bf16; every tile is D/64 TMA boxes of 128
+// rows x 128 bytes with the 128-byte swizzle (the canonical K-major layout
+// for Q and K; V is read as the MN-major B operand of P.V).
 //
 // Every wait is bounded (AttnArgs::timeout_ns).  A wait that runs out sets
 // the device error word and a CTA-wide abort flag; every role then leaves its
@@ -42,26 +52,34 @@ namespace rc {
 
 namespace tc {
 constexpr int kThreads = 320;
-constexpr int kNumSlots = 4;
+constexpr int kSoftmaxThreads = 256;
+constexpr int kNumSlots = 5;
 constexpr int kTileRows = 128;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kBoxBytes = 128 * 128;  // one TMA box: 128 rows x 128 bytes
+constexpr uint32_t kColS = 0, kColP = 256, kColO = 384;
 
 template <int D>
 struct Smem {
   static constexpr uint32_t kTile = kTileRows * D * 2;
-  static constexpr uint32_t kQ0 = 0;
-  static constexpr uint32_t kQ1 = kTile;
+  static constexpr uint32_t kQ = 0;  // Q buffers 0 and 1
   static constexpr uint32_t kRing = 2 * kTile;
   static constexpr uint32_t kBars = kRing + kNumSlots * kTile;
   // barrier indices
-  static constexpr int kQFull = 0, kQEmpty = 1, kSlotFull = 2, kSlotEmpty = 2 + kNumSlots,
-                       kSFull = 2 + 2 * kNumSlots, kPFull = kSFull + 2, kOFull = kPFull + 2,
-                       kOFree = kOFull + 2, kMmaDone = kOFree + 2, kNumBars = kMmaDone + 1;
-  static constexpr uint32_t kTmemHolder = kBars + 8 * kNumBars;
+  static constexpr int kQFull = 0, kQEmpty = 2, kSlotFull = 4, kSlotEmpty = 4 + kNumSlots,
+                       kSFull = 4 + 2 * kNumSlots, kPFull = kSFull + 2, kOFree = kPFull + 2, kMmaDone = kOFree + 1,
+                       kXchg = kMmaDone + 1, kNumBars = kXchg + 4;
+  // partial row maxima / sums exchanged by the two threads of a row:
+  // float [2 parity][2 halves][128 rows]
+  static constexpr uint32_t kXBuf = kBars + 8 * kNumBars;
+  static constexpr uint32_t kTmemHolder = kXBuf + 2 * 2 * 128 * 4;
   static constexpr uint32_t kAbort = kTmemHolder + 4;
   static constexpr uint32_t kUsed = kAbort + 4;
-  static constexpr uint32_t kDynamic = kUsed + 1024;  // slack to align the base to 1024
+  // bytes requested at launch: slack to align the base to 1024, capped at the
+  // 227 KB a CTA may have (the kernel checks that the aligned layout fits)
+  static constexpr uint32_t kMaxDynamic = 232448;
+  static constexpr uint32_t kDynamic = kUsed + 1024 < kMaxDynamic ? kUsed + 1024 : kMaxDynamic;
+  static_assert(kUsed <= kMaxDynamic, "shared-memory layout too large");
 };
 
 struct Ctl {
@@ -116,6 +134,54 @@ __device__ __forceinline__ TileSrc tile_src(const Task& t, int na, int j) {
   }
   return s;
 }
+
+// Items are enumerated head-major (item = head * n_tasks + task, tasks
+// longest first): CTAs that run at the same time then work on few heads, so
+// the K/V tiles they all stream stay in L2.
+__device__ __forceinline__ void decode_item(const AttnArgs& a, int item, Task& t, int& head) {
+  head = item / a.n_tasks;
+  t = a.tasks[item - head * a.n_tasks];
+}
+
+__device__ __forceinline__ int n_key_tiles(const Task& t, int& na) {
+  na = (t.a_len + kTileRows - 1) / kTileRows;
+  return na + (t.b_len + kTileRows - 1) / kTileRows;
+}
+
+// Position in a CTA's key-tile stream: items blockIdx.x, blockIdx.x + grid,
+// ... with at least one key tile; qi counts those items, t the tiles.
+struct Cursor {
+  Task task;
+  int head, item, qi, j, na, nkv, t;
+  bool valid;
+  __device__ __forceinline__ void seek(const AttnArgs& a) {
+    for (; item < a.n_items; item += gridDim.x) {
+      decode_item(a, item, task, head);
+      nkv = n_key_tiles(task, na);
+      if (nkv > 0) {
+        j = 0;
+        valid = true;
+        return;
+      }
+    }
+    valid = false;
+  }
+  __device__ __forceinline__ void init(const AttnArgs& a) {
+    item = blockIdx.x;
+    qi = 0;
+    t = 0;
+    seek(a);
+  }
+  __device__ __forceinline__ bool last_of_item() const { return j == nkv - 1; }
+  __device__ __forceinline__ void advance(const AttnArgs& a) {
+    ++t;
+    if (++j == nkv) {
+      item += gridDim.x;
+      ++qi;
+      seek(a);
+    }
+  }
+};
 }  // namespace tc
 
 template <int D>
@@ -140,20 +206,24 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  if (base - raw + L::kUsed > L::kDynamic) {  // the allocation cannot hold the aligned layout
+    if (threadIdx.x == 0) atomicCAS(&g_rc_status, 0, RC_DEV_TIMEOUT_BASE + 99);
+    return;
+  }
 
   if (threadIdx.x == 0) {
-    mbar_init(bar(L::kQFull), 1);
-    mbar_init(bar(L::kQEmpty), 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(bar(L::kQFull + i), 1);
+      mbar_init(bar(L::kQEmpty + i), 1);
+      mbar_init(bar(L::kSFull + i), 1);
+      mbar_init(bar(L::kPFull + i), kSoftmaxThreads);
+    }
     for (int s = 0; s < kNumSlots; ++s) {
       mbar_init(bar(L::kSlotFull + s), 1);
       mbar_init(bar(L::kSlotEmpty + s), 1);
     }
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(bar(L::kSFull + i), 1);
-      mbar_init(bar(L::kPFull + i), 128);
-      mbar_init(bar(L::kOFull + i), 1);
-      mbar_init(bar(L::kOFree + i), 128);
-    }
+    mbar_init(bar(L::kOFree), kSoftmaxThreads);
+    for (int q = 0; q < 4; ++q) mbar_init(bar(L::kXchg + q), 64);  // warps q and q + 4
     mbar_init(bar(L::kMmaDone), 1);
     *abort_flag = 0;
     fence_barrier_init();
@@ -171,117 +241,156 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
 
   if (warp == 8) {
     // ------------------------------------------------------------ producer
+    // Ring order = the MMA thread's order of use: K_0, K_1, then V_t, K_t+2
+    // for t = 0, 1, ...; an item's Q tile goes out just before its first K.
     if (lane == 0) {
-      uint32_t use = 0, q_uses = 0;
+      uint32_t use = 0;
       int armed_round[kNumSlots];
       for (int s = 0; s < kNumSlots; ++s) armed_round[s] = -1;
-      int q_armed = -1;
+      int q_armed[2] = {-1, -1};
       bool skip_next = args.dbg_skip_first_load != 0;
-      for (int item = blockIdx.x; item < args.n_items; item += gridDim.x) {
-        const Task t = args.tasks[item / args.num_heads];
-        const int head = item % args.num_heads;
-        const int na = (t.a_len + kTileRows - 1) / kTileRows;
-        const int nkv = na + (t.b_len + kTileRows - 1) / kTileRows;
-        if (nkv == 0) continue;
-        const bool two = t.q_rows > kTileRows;
-        if (!wait_one(bar(L::kQEmpty), (q_uses & 1u) ^ 1u, ctl, 1)) goto producer_done;
-        mbar_arrive_expect_tx(bar(L::kQFull), (two ? 2u : 1u) * L::kTile);
-        for (int c = 0; c < kChunks; ++c) {
-          tma_load_2d(base + L::kQ0 + c * kBoxBytes, &tm_q, bar(L::kQFull), head * D + c * 64, t.q_row0);
-          if (two)
-            tma_load_2d(base + L::kQ1 + c * kBoxBytes, &tm_q, bar(L::kQFull), head * D + c * 64,
-                        t.q_row0 + kTileRows);
+      Cursor kc, vc;
+      kc.init(args);
+      vc.init(args);
+      // load K (kv = 0) or V (kv = 1) of the tile at cursor c into the next ring slot
+      auto load_tile = [&](const Cursor& c, int kv) -> bool {
+        const int slot = static_cast<int>(use % kNumSlots);
+        const uint32_t round = use / kNumSlots;
+        ++use;
+        if (!wait_one(bar(L::kSlotEmpty + slot), (round & 1u) ^ 1u, ctl, 2)) return false;
+        if (kv == 0 && skip_next) {  // fault injection: this load never arrives
+          skip_next = false;
+          return true;
         }
-        q_armed = static_cast<int>(q_uses);
-        ++q_uses;
-        for (int j = 0; j < nkv; ++j) {
-          const TileSrc src = tile_src(t, na, j);
-          for (int kv = 0; kv < 2; ++kv, ++use) {
-            const int slot = static_cast<int>(use % kNumSlots);
-            const uint32_t round = use / kNumSlots;
-            if (!wait_one(bar(L::kSlotEmpty + slot), (round & 1u) ^ 1u, ctl, 2)) goto producer_done;
-            if (skip_next) {  // fault injection: this load never arrives
-              skip_next = false;
-              continue;
-            }
-            const void* map = kv == 0 ? (src.in_b ? &tm_kb : &tm_ka) : (src.in_b ? &tm_vb : &tm_va);
-            const uint32_t dst = base + L::kRing + static_cast<uint32_t>(slot) * L::kTile;
-            mbar_arrive_expect_tx(bar(L::kSlotFull + slot), L::kTile);
-            for (int c = 0; c < kChunks; ++c)
-              tma_load_2d(dst + c * kBoxBytes, map, bar(L::kSlotFull + slot), head * D + c * 64, src.row);
-            armed_round[slot] = static_cast<int>(round);
-          }
+        const TileSrc src = tile_src(c.task, c.na, c.j);
+        const void* map = kv == 0 ? (src.in_b ? &tm_kb : &tm_ka) : (src.in_b ? &tm_vb : &tm_va);
+        const uint32_t dst = base + L::kRing + static_cast<uint32_t>(slot) * L::kTile;
+        mbar_arrive_expect_tx(bar(L::kSlotFull + slot), L::kTile);
+        for (int ch = 0; ch < kChunks; ++ch)
+          tma_load_2d(dst + ch * kBoxBytes, map, bar(L::kSlotFull + slot), c.head * D + ch * 64, src.row);
+        armed_round[slot] = static_cast<int>(round);
+        return true;
+      };
+      auto load_k = [&]() -> bool {
+        if (kc.j == 0) {  // the item's Q tile into buffer qi % 2
+          const int b = kc.qi & 1;
+          const uint32_t u = static_cast<uint32_t>(kc.qi >> 1);
+          if (!wait_one(bar(L::kQEmpty + b), (u & 1u) ^ 1u, ctl, 1)) return false;
+          mbar_arrive_expect_tx(bar(L::kQFull + b), L::kTile);
+          for (int ch = 0; ch < kChunks; ++ch)
+            tma_load_2d(base + L::kQ + b * L::kTile + ch * kBoxBytes, &tm_q, bar(L::kQFull + b),
+                        kc.head * D + ch * 64, kc.task.q_row0);
+          q_armed[b] = static_cast<int>(u);
         }
+        if (!load_tile(kc, 0)) return false;
+        kc.advance(args);
+        return true;
+      };
+      for (int n = 0; n < 2 && kc.valid; ++n)
+        if (!load_k()) goto producer_done;
+      while (vc.valid) {
+        if (!load_tile(vc, 1)) goto producer_done;
+        vc.advance(args);
+        if (kc.valid && !load_k()) goto producer_done;
       }
     producer_done:
       // Let every TMA load this CTA issued land before the CTA may exit.
       for (int s = 0; s < kNumSlots; ++s)
         if (armed_round[s] >= 0)
           drain_one(bar(L::kSlotFull + s), static_cast<uint32_t>(armed_round[s]) & 1u, args.timeout_ns);
-      if (q_armed >= 0) drain_one(bar(L::kQFull), static_cast<uint32_t>(q_armed) & 1u, args.timeout_ns);
+      for (int b = 0; b < 2; ++b)
+        if (q_armed[b] >= 0) drain_one(bar(L::kQFull + b), static_cast<uint32_t>(q_armed[b]) & 1u, args.timeout_ns);
     }
     __syncwarp();
   } else if (warp == 9) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      uint32_t use = 0, q_uses = 0;
-      uint32_t p_cnt[2] = {0u, 0u}, ofree_cnt[2] = {0u, 0u};
-      bool ofree_pending[2] = {false, false};
+      uint32_t use = 0;
       bool issued_any = false;
-      for (int item = blockIdx.x; item < args.n_items; item += gridDim.x) {
-        const Task t = args.tasks[item / args.num_heads];
-        const int na = (t.a_len + kTileRows - 1) / kTileRows;
-        const int nkv = na + (t.b_len + kTileRows - 1) / kTileRows;
-        if (nkv == 0) continue;
-        const int ntiles = t.q_rows > kTileRows ? 2 : 1;
-        if (!wait_one(bar(L::kQFull), q_uses & 1u, ctl, 3)) goto mma_done;
-        ++q_uses;
+      Cursor sc, pc;  // S side (two tiles ahead) and P.V side of the stream
+      sc.init(args);
+      pc.init(args);
+      const uint64_t qdesc0 = sdesc_sw128(base + L::kQ, 16, 1024);
+      // wait for the next ring slot to be full; returns its index or -1
+      auto next_slot = [&](int where) -> int {
+        const int slot = static_cast<int>(use % kNumSlots);
+        const uint32_t round = use / kNumSlots;
+        ++use;
+        return wait_one(bar(L::kSlotFull + slot), round & 1u, ctl, where) ? slot : -1;
+      };
+      // the first S of an item waits for the item's Q tile
+      auto wait_q = [&](const Cursor& c) -> bool {
+        if (c.j != 0) return true;
+        return wait_one(bar(L::kQFull + (c.qi & 1)), static_cast<uint32_t>(c.qi >> 1) & 1u, ctl, 3);
+      };
+      // prologue: S_0 and S_1 on their own
+      for (int n = 0; n < 2 && sc.valid; ++n) {
+        if (!wait_q(sc)) goto mma_done;
+        const int ks = next_slot(4);
+        if (ks < 0) goto mma_done;
         tc_fence_after();
-        for (int j = 0; j < nkv; ++j) {
-          const int kslot = static_cast<int>(use % kNumSlots);
-          const uint32_t kround = use / kNumSlots;
-          ++use;
-          const int vslot = static_cast<int>(use % kNumSlots);
-          const uint32_t vround = use / kNumSlots;
-          ++use;
-          if (!wait_one(bar(L::kSlotFull + kslot), kround & 1u, ctl, 4)) goto mma_done;
-          tc_fence_after();
-          const uint32_t kaddr = base + L::kRing + static_cast<uint32_t>(kslot) * L::kTile;
-          for (int i = 0; i < ntiles; ++i) {
-            const uint32_t qaddr = base + (i == 0 ? L::kQ0 : L::kQ1);
+        const uint64_t qd = qdesc0 + ((static_cast<uint32_t>(sc.qi & 1) * L::kTile) >> 4);
+        const uint64_t kd = sdesc_sw128(base + L::kRing + static_cast<uint32_t>(ks) * L::kTile, 16, 1024);
+        const uint32_t d_s = tmem + kColS + 128u * static_cast<uint32_t>(sc.t & 1);
 #pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t off = static_cast<uint32_t>(kk / 4) * kBoxBytes + static_cast<uint32_t>(kk % 4) * 32u;
-              tc_mma_ss(tmem + 128u * i, sdesc_sw128(qaddr + off, 16, 1024), sdesc_sw128(kaddr + off, 16, 1024),
-                        kIdescS, kk > 0 ? 1u : 0u);
-            }
-            tc_commit(bar(L::kSFull + i));
-          }
-          issued_any = true;
-          tc_commit(bar(L::kSlotEmpty + kslot));
-          if (j == nkv - 1) tc_commit(bar(L::kQEmpty));
-          if (!wait_one(bar(L::kSlotFull + vslot), vround & 1u, ctl, 5)) goto mma_done;
-          const uint32_t vaddr = base + L::kRing + static_cast<uint32_t>(vslot) * L::kTile;
-          for (int i = 0; i < ntiles; ++i) {
-            if (j == 0 && ofree_pending[i]) {
-              if (!wait_one(bar(L::kOFree + i), ofree_cnt[i] & 1u, ctl, 6)) goto mma_done;
-              ++ofree_cnt[i];
-              ofree_pending[i] = false;
-            }
-            if (!wait_one(bar(L::kPFull + i), p_cnt[i] & 1u, ctl, 7)) goto mma_done;
-            ++p_cnt[i];
-            tc_fence_after();
-#pragma unroll
-            for (int kk = 0; kk < kTileRows / 16; ++kk) {
-              tc_mma_ts(tmem + 256u + 128u * i, tmem + 128u * i + 8u * kk,
-                        sdesc_sw128(vaddr + 2048u * kk, kBoxBytes, 1024), kIdescO,
-                        (j > 0 || kk > 0) ? 1u : 0u);
-            }
-            tc_commit(bar(L::kOFull + i));
-          }
-          tc_commit(bar(L::kSlotEmpty + vslot));
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint64_t off = (static_cast<uint32_t>(kk >> 2) * kBoxBytes + static_cast<uint32_t>(kk & 3) * 32u) >> 4;
+          tc_mma_ss(d_s, qd + off, kd + off, kIdescS, kk > 0 ? 1u : 0u);
         }
-        for (int i = 0; i < ntiles; ++i) ofree_pending[i] = true;
+        issued_any = true;
+        tc_commit(bar(L::kSlotEmpty + ks));
+        if (sc.last_of_item()) tc_commit(bar(L::kQEmpty + (sc.qi & 1)));
+        tc_commit(bar(L::kSFull + (sc.t & 1)));
+        sc.advance(args);
+      }
+      // pairs: O += P_t V_t interleaved with S_t+2 = Q K_t+2^T
+      while (pc.valid) {
+        const int t = pc.t;
+        const int vs = next_slot(5);
+        if (vs < 0) goto mma_done;
+        if (pc.j == 0 && pc.qi > 0)  // the previous item's epilogue has read O
+          if (!wait_one(bar(L::kOFree), static_cast<uint32_t>(pc.qi - 1) & 1u, ctl, 6)) goto mma_done;
+        if (!wait_one(bar(L::kPFull + (t & 1)), static_cast<uint32_t>(t >> 1) & 1u, ctl, 7)) goto mma_done;
+        const bool has_s = sc.valid;
+        int ks = -1;
+        if (has_s) {
+          if (!wait_q(sc)) goto mma_done;
+          ks = next_slot(4);
+          if (ks < 0) goto mma_done;
+        }
+        tc_fence_after();
+        const uint64_t vd = sdesc_sw128(base + L::kRing + static_cast<uint32_t>(vs) * L::kTile, kBoxBytes, 1024);
+        const uint32_t a_p = tmem + kColP + 64u * static_cast<uint32_t>(t & 1);
+        const uint32_t first = pc.j == 0 ? 1u : 0u;
+        if (has_s) {
+          const uint64_t qd = qdesc0 + ((static_cast<uint32_t>(sc.qi & 1) * L::kTile) >> 4);
+          const uint64_t kd = sdesc_sw128(base + L::kRing + static_cast<uint32_t>(ks) * L::kTile, 16, 1024);
+          const uint32_t d_s = tmem + kColS + 128u * static_cast<uint32_t>(t & 1);
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) {
+            // P.V step kk: keys 16 kk .. 16 kk + 15 (2048 bytes of V, 8 TMEM columns of P)
+            tc_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, (first && kk == 0) ? 0u : 1u);
+            if (kk < D / 16) {
+              // S step kk: 64-column box kk / 4, 32-byte slice kk % 4 of its swizzle atoms
+              const uint64_t off =
+                  (static_cast<uint32_t>(kk >> 2) * kBoxBytes + static_cast<uint32_t>(kk & 3) * 32u) >> 4;
+              tc_mma_ss(d_s, qd + off, kd + off, kIdescS, kk > 0 ? 1u : 0u);
+            }
+          }
+        } else {
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk)
+            tc_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, (first && kk == 0) ? 0u : 1u);
+        }
+        tc_commit(bar(L::kSlotEmpty + vs));
+        if (has_s) {
+          tc_commit(bar(L::kSlotEmpty + ks));
+          if (sc.last_of_item()) tc_commit(bar(L::kQEmpty + (sc.qi & 1)));
+          sc.advance(args);
+        }
+        // buffer t % 2: S_t+2 is ready and pair t (hence O += P_t V_t) is complete
+        tc_commit(bar(L::kSFull + (t & 1)));
+        pc.advance(args);
       }
     mma_done:
       if (issued_any) {  // every MMA issued must finish before TMEM is freed
@@ -291,125 +400,148 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
     }
     __syncwarp();
   } else {
-    // ------------------------------------------------------------ softmax groups
-    const int grp = warp >> 2;               // query tile of this group
-    const int trow = threadIdx.x & 127;      // row within the tile (= TMEM lane)
-    const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
-    const uint32_t t_s = tmem + lane_off + 128u * grp;
-    const uint32_t t_o = tmem + lane_off + 256u + 128u * grp;
+    // ------------------------------------------------------------ softmax
+    // s_full[b] phase p completes when S of tile 2p + b is in buffer b; phase
+    // p + 1 also means pair 2p + b (O += P V of that tile) is complete.
+    const int quarter = warp & 3;
+    const int half = warp >> 2;                 // score columns [64 half, 64 half + 64)
+    const int trow = quarter * 32 + lane;       // row of the query tile (= TMEM lane)
+    const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
+    const uint32_t col0 = 64u * static_cast<uint32_t>(half);
+    constexpr int kOCols = D / 2;               // O columns this thread rescales / stores
     const float sl2 = args.scale_log2;
-    uint32_t s_cnt = 0, o_cnt = 0;
+    float* xbuf = reinterpret_cast<float*>(base_ptr + L::kXBuf);
+    const uint32_t xbar = bar(L::kXchg + quarter);
+    uint32_t x_phase = 0;                       // exchanges done with the partner thread
+    uint32_t s_waited[2] = {0u, 0u};            // phases of s_full[b] already waited for
+    int t = 0;                                  // position in the key-tile stream
+    // wait until phase `ph` of s_full[b] has completed (each phase once, in order)
+    auto wait_s = [&](int b, uint32_t ph, int where) -> bool {
+      if (s_waited[b] > ph) return true;
+      if (!wait_warp(bar(L::kSFull + b), ph & 1u, ctl, where)) return false;
+      s_waited[b] = ph + 1;
+      return true;
+    };
+    // combine a value with the partner thread's (the other half of the row)
+    auto exchange = [&](float v, float& other, int where) -> bool {
+      float* slot = xbuf + (x_phase & 1u) * 256;
+      slot[half * 128 + trow] = v;
+      mbar_arrive(xbar);
+      if (!wait_warp(xbar, x_phase & 1u, ctl, where)) return false;
+      other = slot[(half ^ 1) * 128 + trow];
+      ++x_phase;
+      return true;
+    };
     for (int item = blockIdx.x; item < args.n_items; item += gridDim.x) {
-      const Task t = args.tasks[item / args.num_heads];
-      const int head = item % args.num_heads;
-      if (grp == 1 && t.q_rows <= kTileRows) continue;
-      const int na = (t.a_len + kTileRows - 1) / kTileRows;
-      const int nkv = na + (t.b_len + kTileRows - 1) / kTileRows;
-      const int row = grp * kTileRows + trow;
-      const bool row_ok = row < t.q_rows;
-      const int64_t grow = static_cast<int64_t>(t.q_row0) + row;
-      __nv_bfloat16* orow = args.out + grow * args.row_stride + static_cast<int64_t>(head) * D;
+      Task tk;
+      int head;
+      decode_item(args, item, tk, head);
+      int na;
+      const int nkv = n_key_tiles(tk, na);
+      const bool row_ok = trow < tk.q_rows;
+      const int64_t grow = static_cast<int64_t>(tk.q_row0) + trow;
+      __nv_bfloat16* orow = args.out + grow * args.row_stride + static_cast<int64_t>(head) * D + half * kOCols;
       if (nkv == 0) {
         if (row_ok) {
           uint4 z = make_uint4(0, 0, 0, 0);
-          for (int c = 0; c < D / 8; ++c) reinterpret_cast<uint4*>(orow)[c] = z;
-          if (args.lse) args.lse[grow * args.num_heads + head] = -INFINITY;
+          for (int c = 0; c < kOCols / 8; ++c) reinterpret_cast<uint4*>(orow)[c] = z;
+          if (args.lse && half == 0) args.lse[grow * args.num_heads + head] = -INFINITY;
         }
         continue;
       }
-      float m_run = 0.f, l_run = 0.f;
-      for (int j = 0; j < nkv; ++j) {
-        const TileSrc src = tile_src(t, na, j);
-        if (!wait_warp(bar(L::kSFull + grp), s_cnt & 1u, ctl, 8)) goto softmax_done;
-        ++s_cnt;
+      float m_run = 0.f, l_run = 0.f;  // l_run: this thread's half of the row sum
+      for (int j = 0; j < nkv; ++j, ++t) {
+        const int b = t & 1;
+        const TileSrc src = tile_src(tk, na, j);
+        if (!wait_s(b, static_cast<uint32_t>(t >> 1), 8)) goto softmax_done;
         tc_fence_after();
-        uint32_t r0[32], r1[32], r2[32], r3[32];
+        const uint32_t t_s = tmem + lane_off + kColS + 128u * b + col0;
+        uint32_t r0[32], r1[32];
         tmem_ld32(t_s + 0u, r0);
         tmem_ld32(t_s + 32u, r1);
-        tmem_ld32(t_s + 64u, r2);
-        tmem_ld32(t_s + 96u, r3);
         tmem_wait_ld(r0);
         tmem_wait_ld(r1);
-        tmem_wait_ld(r2);
-        tmem_wait_ld(r3);
-        float s[128];
+        float s[64];
 #pragma unroll
         for (int c = 0; c < 32; ++c) {
           s[c] = __uint_as_float(r0[c]);
           s[32 + c] = __uint_as_float(r1[c]);
-          s[64 + c] = __uint_as_float(r2[c]);
-          s[96 + c] = __uint_as_float(r3[c]);
         }
-        if (src.valid < kTileRows) {
+        const int valid = src.valid - static_cast<int>(col0);  // keys of this half inside the range
+        if (valid < 64) {
 #pragma unroll
-          for (int c = 0; c < 128; ++c)
-            if (c >= src.valid) s[c] = -INFINITY;
+          for (int c = 0; c < 64; ++c)
+            if (c >= valid) s[c] = -INFINITY;
         }
-        float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
+        // this half's maximum as a tree (depth 6), then the whole row's
+        float mx[32];
 #pragma unroll
-        for (int c = 4; c < 128; c += 4) {
-          mx0 = fmaxf(mx0, s[c]);
-          mx1 = fmaxf(mx1, s[c + 1]);
-          mx2 = fmaxf(mx2, s[c + 2]);
-          mx3 = fmaxf(mx3, s[c + 3]);
-        }
-        const float m_tile = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;
-        if (j > 0) {
-          // O_i holds P_{j-1} V_{j-1} once S_i of tile j is complete; this
-          // wait keeps the phase count in step and returns at once.
-          if (!wait_warp(bar(L::kOFull + grp), o_cnt & 1u, ctl, 9)) goto softmax_done;
-          ++o_cnt;
-          tc_fence_after();
-          const bool need = m_tile > m_run + 8.0f;
-          if (__any_sync(0xffffffffu, need)) {
-            const float m_new = fmaxf(m_run, m_tile);
-            const float alpha = ex2_approx(m_run - m_new);
-            m_run = m_new;
-            l_run *= alpha;
+        for (int c = 0; c < 32; ++c) mx[c] = fmaxf(s[c], s[c + 32]);
 #pragma unroll
-            for (int cc = 0; cc < D / 16; ++cc) {
-              uint32_t o[16];
-              tmem_ld16(t_o + 16u * cc, o);
-              tmem_wait_ld(o);
+        for (int w = 16; w >= 1; w >>= 1)
 #pragma unroll
-              for (int c = 0; c < 16; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * alpha);
-              tmem_st16(t_o + 16u * cc, o);
-            }
-          }
-        } else {
+          for (int c = 0; c < w; ++c) mx[c] = fmaxf(mx[c], mx[c + w]);
+        float mo;
+        if (!exchange(mx[0], mo, 11)) goto softmax_done;
+        const float m_tile = fmaxf(mx[0], mo) * sl2;
+        if (j == 0) {
           m_run = m_tile;
-        }
-        // P = exp2(scaled S - m) as bf16 pairs, written 16 score columns
-        // (8 TMEM columns) at a time over the S columns already consumed.
-        const float neg_m = -m_run;
-        float ls0 = 0.f, ls1 = 0.f;
+        } else if (__any_sync(0xffffffffu, m_tile > m_run + 8.0f)) {
+          // both threads of a row see the same m_tile, so warps q and q + 4 decide alike.
+          // Move the running maximum: O must first hold P_{t-1} V_{t-1}
+          // (pair t-1 complete = phase (t+1)/2 of s_full[(t+1) % 2])
+          if (!wait_s((t + 1) & 1, static_cast<uint32_t>((t + 1) >> 1), 9)) goto softmax_done;
+          tc_fence_after();
+          const float m_new = fmaxf(m_run, m_tile);
+          const float alpha = ex2_approx(m_run - m_new);
+          m_run = m_new;
+          l_run *= alpha;
+          const uint32_t t_o = tmem + lane_off + kColO + static_cast<uint32_t>(half * kOCols);
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
+          for (int cc = 0; cc < kOCols / 16; ++cc) {
+            uint32_t o[16];
+            tmem_ld16(t_o + 16u * cc, o);
+            tmem_wait_ld(o);
+#pragma unroll
+            for (int c = 0; c < 16; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * alpha);
+            tmem_st16(t_o + 16u * cc, o);
+          }
+        }
+        // P = exp2(scaled S - m) as bf16 pairs into P buffer b (this half: 32 columns)
+        const float neg_m = -m_run;
+        const uint32_t t_p = tmem + lane_off + kColP + 64u * b + 32u * static_cast<uint32_t>(half);
+        float ls[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
           uint32_t pk[8];
 #pragma unroll
           for (int c = 0; c < 8; ++c) {
-            const float a = ex2_approx(fmaf(s[16 * q + 2 * c], sl2, neg_m));
-            const float b = ex2_approx(fmaf(s[16 * q + 2 * c + 1], sl2, neg_m));
-            ls0 += a;
-            ls1 += b;
-            pk[c] = pack_bf16x2(a, b);
+            const float x = ex2_approx(fmaf(s[16 * q + 2 * c], sl2, neg_m));
+            const float y = ex2_approx(fmaf(s[16 * q + 2 * c + 1], sl2, neg_m));
+            ls[(2 * c) & 3] += x;
+            ls[(2 * c + 1) & 3] += y;
+            pk[c] = pack_bf16x2(x, y);
           }
-          tmem_st8(t_s + 8u * q, pk);
+          tmem_st8(t_p + 8u * q, pk);
         }
-        l_run += ls0 + ls1;
+        l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
         tmem_wait_st();
         tc_fence_before();
-        mbar_arrive(bar(L::kPFull + grp));
+        mbar_arrive(bar(L::kPFull + b));
       }
-      // epilogue: O_i / l -> bf16 rows
-      if (!wait_warp(bar(L::kOFull + grp), o_cnt & 1u, ctl, 10)) goto softmax_done;
-      ++o_cnt;
-      tc_fence_after();
+      // epilogue: wait for the item's last pair, then O / l -> bf16 rows
       {
-        const float inv_l = 1.0f / l_run;
-        uint32_t packed[D / 2];
+        float l_other;
+        if (!exchange(l_run, l_other, 12)) goto softmax_done;
+        const float l_row = l_run + l_other;
+        const int tl = t - 1;
+        if (!wait_s(tl & 1, static_cast<uint32_t>(tl >> 1) + 1u, 10)) goto softmax_done;
+        tc_fence_after();
+        const float inv_l = 1.0f / l_row;
+        const uint32_t t_o = tmem + lane_off + kColO + static_cast<uint32_t>(half * kOCols);
+        uint32_t packed[kOCols / 2];
 #pragma unroll
-        for (int cc = 0; cc < D / 32; ++cc) {
+        for (int cc = 0; cc < kOCols / 32; ++cc) {
           uint32_t o[32];
           tmem_ld32(t_o + 32u * cc, o);
           tmem_wait_ld(o);
@@ -419,14 +551,14 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
                 pack_bf16x2(__uint_as_float(o[2 * c]) * inv_l, __uint_as_float(o[2 * c + 1]) * inv_l);
         }
         tc_fence_before();
-        mbar_arrive(bar(L::kOFree + grp));
+        mbar_arrive(bar(L::kOFree));
         if (row_ok) {
           uint4* dst = reinterpret_cast<uint4*>(orow);
 #pragma unroll
-          for (int c = 0; c < D / 8; ++c)
+          for (int c = 0; c < kOCols / 8; ++c)
             dst[c] = make_uint4(packed[4 * c], packed[4 * c + 1], packed[4 * c + 2], packed[4 * c + 3]);
-          if (args.lse)
-            args.lse[grow * args.num_heads + head] = (m_run + log2f(l_run)) * 0.69314718055994530942f;
+          if (args.lse && half == 0)
+            args.lse[grow * args.num_heads + head] = (m_run + log2f(l_row)) * 0.69314718055994530942f;
         }
       }
     }

@@ -176,6 +176,20 @@ __device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8])
 #undef RC_P8
 #undef RC_S8
 
+// ---------------------------------------------------------------- register split
+// Warpgroup-wide (all four warps execute it): lower / raise this warp's
+// register allocation.  `inc` waits until the CTA's pool (threads x registers
+// at launch) has the registers, so the shares of all warpgroups must add up
+// to no more than that pool -- the launcher checks it before every launch.
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_inc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_dec() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
+
 // ---------------------------------------------------------------- descriptors
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, bool b_mn_major) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |

@@ -119,7 +119,7 @@ int make_tmap(CUtensorMap* m, const void* base, int64_t rows, int H, int D) {
 }
 
 // ---------------------------------------------------------------- work lists
-constexpr int kTaskRows = 256;
+constexpr int kTaskRows = 128;  // query rows per task (the tcgen05 kernel's tile)
 
 void add_rows(std::vector<Task>& v, int q0, int qn, int a0, int an, int b0, int bn) {
   for (int r = 0; r < qn; r += kTaskRows) {
@@ -195,7 +195,7 @@ int launch_mma(const AttnArgs& a, DeviceInfo* info, cudaStream_t s) {
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_mma_kernel)");
     info->attr_set[key] = true;
   }
-  rc::attn_mma_kernel<D><<<a.n_items * 4, 128, smem, s>>>(a);
+  rc::attn_mma_kernel<D><<<a.n_items * 2, 128, smem, s>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "attn_mma_kernel launch");
   return REFCACHE_OK;
@@ -592,7 +592,7 @@ int full_attention_noalloc(int batch, int num_heads, int head_dim, const int32_t
   for (int b = 0; b < batch; ++b) n_tasks += (cu_seqlens[b + 1] - cu_seqlens[b] + kTaskRows - 1) / kTaskRows;
   if (n_tasks > REFCACHE_NOALLOC_MAX_TASKS)
     return fail(REFCACHE_ERR_INVALID_ARG,
-                "full_attention_noalloc: %lld work items exceed the static limit of %d (256 query rows each)",
+                "full_attention_noalloc: %lld work items exceed the static limit of %d (128 query rows each)",
                 static_cast<long long>(n_tasks), REFCACHE_NOALLOC_MAX_TASKS);
   const int64_t rows = cu_seqlens[batch];
   if ((rc = check_ptrs({q, k, v, o}, rows, "full_attention_noalloc")) != 0) return rc;

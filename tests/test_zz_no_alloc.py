@@ -56,7 +56,7 @@ def test_noalloc_matches_full_attention_twice(kernel):
 
 def test_noalloc_rejects_inputs_beyond_its_limit():
     lib = rcb.load()
-    rows = (rcb.NOALLOC_MAX_TASKS + 1) * 256
+    rows = (rcb.NOALLOC_MAX_TASKS + 1) * 128
     cu = (ctypes.c_int32 * 2)(0, rows)
     q = torch.empty(16, dtype=torch.bfloat16, device="cuda")
     rc = lib.full_attention_noalloc(1, 1, 64, cu, q.data_ptr(), q.data_ptr(), q.data_ptr(), q.data_ptr(), None,
