@@ -3,8 +3,8 @@
 // "recompiled pre-Blackwell kernel" comparison point for the tcgen05 kernel.
 //
 // CTA = 4 warps = 64 query rows (16 per warp) of one (task, head) item;
-// blockIdx.x = 2 * item + sub, sub selecting rows [64 sub, 64 sub + 64) of
-// the task (tasks hold at most 128 rows).  Key tiles of 64 rows stream through a double-buffered cp.async
+// blockIdx.x = (rows_per_task / 64) * item + sub, sub selecting rows
+// [64 sub, 64 sub + 64) of the task.  Key tiles of 64 rows stream through a double-buffered cp.async
 // pipeline (range A, then range B); scores, online softmax (exact running
 // maximum, fp32) and the P.V accumulation stay in registers.
 #pragma once
@@ -65,7 +65,8 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a) {
   // element offset of (row, 16-byte chunk) with the chunk XOR-swizzled by row
   auto off = [](int row, int ch) { return row * D + ((ch ^ (row & 7)) << 3); };
 
-  const int item = blockIdx.x >> 1, sub = blockIdx.x & 1;
+  const int per_task = a.rows_per_task / 64;
+  const int item = blockIdx.x / per_task, sub = blockIdx.x % per_task;
   if (item >= a.n_items) return;
   const Task t = a.tasks[item / a.num_heads];
   const int head = item % a.num_heads;

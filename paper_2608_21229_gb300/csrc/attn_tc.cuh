@@ -148,14 +148,14 @@ __device__ __forceinline__ int n_key_tiles(const Task& t, int& na) {
   return na + (t.b_len + kTileRows - 1) / kTileRows;
 }
 
-// Position in a CTA's key-tile stream: items blockIdx.x, blockIdx.x + grid,
-// ... with at least one key tile; qi counts those items, t the tiles.
+// Position in a CTA's key-tile stream: items first, first + stride, ...
+// with at least one key tile; qi counts those items, t the tiles.
 struct Cursor {
   Task task;
-  int head, item, qi, j, na, nkv, t;
+  int head, item, stride, qi, j, na, nkv, t;
   bool valid;
   __device__ __forceinline__ void seek(const AttnArgs& a) {
-    for (; item < a.n_items; item += gridDim.x) {
+    for (; item < a.n_items; item += stride) {
       decode_item(a, item, task, head);
       nkv = n_key_tiles(task, na);
       if (nkv > 0) {
@@ -166,8 +166,9 @@ struct Cursor {
     }
     valid = false;
   }
-  __device__ __forceinline__ void init(const AttnArgs& a) {
-    item = blockIdx.x;
+  __device__ __forceinline__ void init(const AttnArgs& a, int first, int step) {
+    item = first;
+    stride = step;
     qi = 0;
     t = 0;
     seek(a);
@@ -176,7 +177,7 @@ struct Cursor {
   __device__ __forceinline__ void advance(const AttnArgs& a) {
     ++t;
     if (++j == nkv) {
-      item += gridDim.x;
+      item += stride;
       ++qi;
       seek(a);
     }
@@ -250,8 +251,8 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
       int q_armed[2] = {-1, -1};
       bool skip_next = args.dbg_skip_first_load != 0;
       Cursor kc, vc;
-      kc.init(args);
-      vc.init(args);
+      kc.init(args, blockIdx.x, gridDim.x);
+      vc.init(args, blockIdx.x, gridDim.x);
       // load K (kv = 0) or V (kv = 1) of the tile at cursor c into the next ring slot
       auto load_tile = [&](const Cursor& c, int kv) -> bool {
         const int slot = static_cast<int>(use % kNumSlots);
@@ -308,8 +309,8 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
       uint32_t use = 0;
       bool issued_any = false;
       Cursor sc, pc;  // S side (two tiles ahead) and P.V side of the stream
-      sc.init(args);
-      pc.init(args);
+      sc.init(args, blockIdx.x, gridDim.x);
+      pc.init(args, blockIdx.x, gridDim.x);
       const uint64_t qdesc0 = sdesc_sw128(base + L::kQ, 16, 1024);
       // wait for the next ring slot to be full; returns its index or -1
       auto next_slot = [&](int where) -> int {

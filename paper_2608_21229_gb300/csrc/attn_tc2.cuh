@@ -1,0 +1,506 @@
+// attn_tc2.cuh -- the head_dim-128 attention kernel on CTA pairs: the same
+// computation and pair schedule as attn_tc.cuh, with every MMA issued over
+// two CTAs on neighbouring SMs (tcgen05 cta_group::2, M = 256).
+//
+// Why pairs: with one 128-row query tile per SM, each S/P.V pair of MMAs
+// (1024 tensor cycles) needs a fresh 32 KB K tile and 32 KB V tile in that
+// SM's shared memory.  The tensor core's operand reads (about 96 KB per pair)
+// plus those 64 KB of TMA fills exceed what one SM's shared memory delivers
+// in 1024 cycles (128 bytes per cycle), so the tensor core waits for data.  A
+// CTA pair shares every K/V tile: CTA r holds keys [64 r, 64 r + 64) of each
+// K tile and head-dim columns [64 r, 64 r + 64) of each V tile (the B operand
+// of a cta_group::2 MMA is split along N between the two CTAs), while each
+// CTA keeps its own 128 query rows (A is split along M).  Per SM this halves
+// the tile bytes fetched and the B-operand bytes read, for the same MMA work.
+//
+// Cluster of 2 CTAs (rank 0 = leader), 320 threads each:
+//   warps 0-7  softmax of this CTA's 128 rows (as in attn_tc.cuh)
+//   warp 8     TMA producer: this CTA's Q rows and its halves of the K and V
+//              tiles; completion is counted on the leader's barriers
+//   warp 9     both CTAs: TMEM allocation (a pair operation); leader only:
+//              the MMA thread
+// An item is a task of up to 256 query rows: CTA r takes rows
+// [128 r, 128 r + 128).  Items are taken cluster by cluster, head-major.
+//
+// The key tiles of all items a cluster runs form one stream t = 0 .. T-1.
+// Pair p of MMAs (p = -2, -1: S_0, S_1 alone; p >= 0: O += P_p V_p
+// interleaved, MMA by MMA, with S_p+2 = Q K_p+2^T) reads ring stage u = p + 2,
+// which holds K_u (if u < T) and V_u-2 (if u >= 2); the ring has kStages
+// stages of 32 KB per CTA.
+//
+// Synchronisation is built so that the MMA thread does as little as possible
+// between its MMAs: a tcgen05.mma blocks its thread for about as long as the
+// tensor core takes to run it, and the tensor core queues only a few, so any
+// wait or commit between two MMAs idles the tensor core unless it is short.
+// Per pair the MMA thread waits once (P ready) and commits once:
+//   pair_done[p & 3]   one commit per pair (multicast to both CTAs).  Pair p
+//                      complete means: S_p+2 is in S buffer p % 2, O holds
+//                      P_p V_p, P buffer p % 2 and ring stage p + 2 are free.
+//                      Four barriers, so that no waiter can miss a phase: a
+//                      waiter for pair p holds up pair p + 4.
+//   p_full[t % 2]      one arrival per softmax warp of both CTAs.  Its phase
+//                      for tile t means P_t is in TMEM, every softmax thread
+//                      has finished reading O for the previous item, and (the
+//                      leader's warp 0 waited for it) stage t + 2 is full.
+//   stage_full[s]      the producers' TMA bytes of both CTAs (leader's barrier)
+//   q_full / q_empty   per Q buffer, once per item
+#pragma once
+#include "attn_tc.cuh"
+
+namespace rc {
+
+namespace tc2 {
+using tc::Ctl;
+constexpr int kD = 128;
+constexpr int kThreads = 320;
+constexpr int kStages = 4;                  // ring stages (pair_done has as many barriers)
+constexpr uint32_t kKHalf = 64 * 128 * 2;   // 16 KB: this CTA's 64 keys x 128 d of a K tile
+constexpr uint32_t kVHalf = 128 * 64 * 2;   // 16 KB: 128 keys x this CTA's 64 d of a V tile
+constexpr uint32_t kStage = kKHalf + kVHalf;
+constexpr uint32_t kQTile = 128 * 128 * 2;
+constexpr uint32_t kKBox = 64 * 128;        // one K box: 64 rows x 128 bytes
+constexpr int kWarpArrivals = 16;           // 8 softmax warps in each of the 2 CTAs
+static_assert(kStages == 4, "pair_done indexing assumes four stages");
+
+struct Smem {
+  static constexpr uint32_t kQ = 0;                // Q buffers 0 and 1 (this CTA's 128 rows)
+  static constexpr uint32_t kRing = 2 * kQTile;    // stage s: [K half | V half]
+  static constexpr uint32_t kBars = kRing + kStages * kStage;
+  static constexpr int kQFull = 0, kQEmpty = 2, kStageFull = 4, kPairDone = 4 + kStages, kPFull = kPairDone + 4,
+                       kMmaDone = kPFull + 2, kXchg = kMmaDone + 1, kNumBars = kXchg + 4;
+  static constexpr uint32_t kXBuf = kBars + 8 * kNumBars;
+  static constexpr uint32_t kTmemHolder = kXBuf + 2 * 2 * 128 * 4;
+  static constexpr uint32_t kAbort = kTmemHolder + 4;
+  static constexpr uint32_t kUsed = kAbort + 4;
+  static constexpr uint32_t kMaxDynamic = 232448;
+  static constexpr uint32_t kDynamic = kUsed + 1024 < kMaxDynamic ? kUsed + 1024 : kMaxDynamic;
+  static_assert(kUsed <= kMaxDynamic, "shared-memory layout too large");
+};
+
+// Phase parity of pair_done[p & 3] that completes with pair p (p >= -2).
+__device__ __forceinline__ uint32_t pair_parity(int p) { return static_cast<uint32_t>((p + 2) >> 2) & 1u; }
+
+// Bounded wait with cluster-scope acquire (barriers other CTAs arrive on).
+__device__ __forceinline__ bool wait_cl(uint32_t bar, uint32_t parity, const Ctl& c, int where) {
+  if (mbar_try_wait_cluster(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (;;) {
+    for (int i = 0; i < 16; ++i)
+      if (mbar_try_wait_cluster(bar, parity)) return true;
+    if (*c.abort_flag) return false;
+    if (globaltimer_ns() - t0 > c.timeout_ns) {
+      *c.abort_flag = 1;
+      atomicCAS(&g_rc_status, 0, RC_DEV_TIMEOUT_BASE + where);
+      return false;
+    }
+  }
+}
+__device__ __forceinline__ bool wait_cl_warp(uint32_t bar, uint32_t parity, const Ctl& c, int where) {
+  const bool ok = wait_cl(bar, parity, c, where);
+  return __all_sync(0xffffffffu, ok);
+}
+}  // namespace tc2
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
+    attn_tc2_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_ka,
+                    const __grid_constant__ CUtensorMap tm_va, const __grid_constant__ CUtensorMap tm_kb,
+                    const __grid_constant__ CUtensorMap tm_vb, const AttnArgs args) {
+  using namespace tc;
+  using tc2::kKBox;
+  using tc2::kKHalf;
+  using tc2::kQTile;
+  using tc2::kStage;
+  using tc2::kStages;
+  using tc2::kVHalf;
+  using tc2::kWarpArrivals;
+  using tc2::pair_parity;
+  using tc2::wait_cl;
+  using tc2::wait_cl_warp;
+  using L = tc2::Smem;
+  constexpr int D = tc2::kD;
+  constexpr uint32_t kIdescS = idesc_bf16_f32(256, 128, false);
+  constexpr uint32_t kIdescO = idesc_bf16_f32(256, D, true);
+
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* base_ptr = smem_raw + (base - raw);
+  auto bar = [&](int i) -> uint32_t { return base + L::kBars + 8u * static_cast<uint32_t>(i); };
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(base_ptr + L::kAbort);
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(base_ptr + L::kTmemHolder);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  const int cluster = static_cast<int>(blockIdx.x >> 1);
+  const int n_clusters = static_cast<int>(gridDim.x >> 1);
+  // Both CTAs of a pair get the same layout, so both leave here together.
+  if (base - raw + L::kUsed > L::kDynamic) {
+    if (threadIdx.x == 0) atomicCAS(&g_rc_status, 0, RC_DEV_TIMEOUT_BASE + 99);
+    return;
+  }
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(bar(L::kQFull + i), 1);
+      mbar_init(bar(L::kQEmpty + i), 1);
+      mbar_init(bar(L::kPFull + i), kWarpArrivals);
+    }
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(bar(L::kStageFull + s), 1);
+      mbar_init(bar(L::kPairDone + s), 1);
+    }
+    mbar_init(bar(L::kMmaDone), 1);
+    for (int q = 0; q < 4; ++q) mbar_init(bar(L::kXchg + q), 64);
+    *abort_flag = 0;
+    fence_barrier_init();
+    fence_proxy_async_smem();
+  }
+  if (warp == 9) {
+    tmem_alloc_pair(smem_u32(tmem_holder), kTmemCols);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // both CTAs' barriers exist before any cross-CTA arrival
+  tc_fence_after();
+  const uint32_t tmem = *tmem_holder;
+  const Ctl ctl{abort_flag, args.timeout_ns};
+  auto lbar = [&](int i) -> uint32_t { return mapa_shared(bar(i), 0); };  // leader's barrier i
+
+  if (warp == 8) {
+    // ------------------------------------------------------------ producer (both CTAs)
+    // Stages u = 0 .. T+1 in order: K_u (u < T) and V_u-2 (u >= 2), this
+    // CTA's halves.  Stage 1 of a one-tile stream is empty.  An item's Q rows
+    // go out just before the stage that holds the item's first K tile.
+    if (lane == 0) {
+      int armed_phase[kStages];
+      for (int s = 0; s < kStages; ++s) armed_phase[s] = -1;
+      int q_armed[2] = {-1, -1};
+      bool skip_next = leader && args.dbg_skip_first_load != 0;
+      Cursor kc, vc;
+      kc.init(args, cluster, n_clusters);
+      vc.init(args, cluster, n_clusters);
+      int u = 0;
+      auto load_q = [&]() -> bool {  // this CTA's 128 query rows of kc's item into Q buffer qi % 2
+        const int b = kc.qi & 1;
+        const uint32_t n = static_cast<uint32_t>(kc.qi >> 1);
+        if (!wait_one(bar(L::kQEmpty + b), (n & 1u) ^ 1u, ctl, 1)) return false;
+        if (leader) {
+          mbar_arrive_expect_tx(bar(L::kQFull + b), 2 * kQTile);
+          q_armed[b] = static_cast<int>(n);
+        }
+        const uint32_t qfull = lbar(L::kQFull + b);
+        for (int ch = 0; ch < 2; ++ch)
+          tma_load_2d_pair(base + L::kQ + b * kQTile + ch * kBoxBytes, &tm_q, qfull, kc.head * D + ch * 64,
+                           kc.task.q_row0 + 128 * static_cast<int>(rank));
+        return true;
+      };
+      // stage u: V of vc's tile (if with_v) and K of kc's tile (if with_k)
+      auto load_stage = [&](bool with_v, bool with_k) -> bool {
+        if (with_k && kc.j == 0 && !load_q()) return false;
+        const int slot = u & (kStages - 1);
+        // the stage's previous use (u - kStages) is read by pair u - kStages - 2
+        if (u >= kStages && !wait_one(bar(L::kPairDone + ((u + 2) & 3)), pair_parity(u - kStages - 2), ctl, 2))
+          return false;
+        const uint32_t dst = base + L::kRing + static_cast<uint32_t>(slot) * kStage;
+        const uint32_t full = lbar(L::kStageFull + slot);
+        const uint32_t bytes = 2 * ((with_k ? kKHalf : 0u) + (with_v ? kVHalf : 0u));
+        if (skip_next) {  // fault injection: the leader never arms or loads this stage
+          skip_next = false;
+        } else {
+          if (leader) {
+            mbar_arrive_expect_tx(bar(L::kStageFull + slot), bytes);
+            armed_phase[slot] = (u / kStages) & 1;
+          }
+          if (with_k) {  // keys [64 r, 64 r + 64) of the tile, both head-dim boxes
+            const TileSrc src = tile_src(kc.task, kc.na, kc.j);
+            const void* map = src.in_b ? &tm_kb : &tm_ka;
+            for (int ch = 0; ch < 2; ++ch)
+              tma_load_2d_pair(dst + ch * kKBox, map, full, kc.head * D + ch * 64,
+                               src.row + 64 * static_cast<int>(rank));
+          }
+          if (with_v) {  // head-dim columns [64 r, 64 r + 64) of all 128 keys
+            const TileSrc src = tile_src(vc.task, vc.na, vc.j);
+            const void* map = src.in_b ? &tm_vb : &tm_va;
+            tma_load_2d_pair(dst + kKHalf, map, full, vc.head * D + 64 * static_cast<int>(rank), src.row);
+          }
+        }
+        ++u;
+        return true;
+      };
+      if (kc.valid) {
+        for (int n = 0; n < 2; ++n) {
+          const bool with_k = kc.valid;
+          if (!load_stage(false, with_k)) goto producer_done;
+          if (with_k) kc.advance(args);
+        }
+        while (vc.valid) {
+          const bool with_k = kc.valid;
+          if (!load_stage(true, with_k)) goto producer_done;
+          vc.advance(args);
+          if (with_k) kc.advance(args);
+        }
+      }
+    producer_done:
+      // the leader's full barriers count both CTAs' bytes: once they complete,
+      // every load of the pair has landed
+      for (int s = 0; s < kStages; ++s)
+        if (armed_phase[s] >= 0)
+          drain_one(bar(L::kStageFull + s), static_cast<uint32_t>(armed_phase[s]), args.timeout_ns);
+      for (int b = 0; b < 2; ++b)
+        if (q_armed[b] >= 0) drain_one(bar(L::kQFull + b), static_cast<uint32_t>(q_armed[b]) & 1u, args.timeout_ns);
+    }
+    __syncwarp();
+  } else if (warp == 9) {
+    // ------------------------------------------------------------ MMA issuer (leader)
+    if (leader && lane == 0) {
+      Cursor sc, pc;  // S side (two tiles ahead) and P.V side of the stream
+      sc.init(args, cluster, n_clusters);
+      pc.init(args, cluster, n_clusters);
+      const uint64_t qdesc0 = sdesc_sw128(base + L::kQ, 16, 1024);
+      auto wait_q = [&](const Cursor& c) -> bool {
+        if (c.j != 0) return true;
+        return wait_one(bar(L::kQFull + (c.qi & 1)), static_cast<uint32_t>(c.qi >> 1) & 1u, ctl, 3);
+      };
+      // S step kk: A = Q (128-row boxes of 16 KB), B = this CTA's 64 keys (64-row boxes of 8 KB)
+      auto q_off = [](int kk) -> uint64_t {
+        return (static_cast<uint32_t>(kk >> 2) * kBoxBytes + static_cast<uint32_t>(kk & 3) * 32u) >> 4;
+      };
+      auto k_off = [](int kk) -> uint64_t {
+        return (static_cast<uint32_t>(kk >> 2) * kKBox + static_cast<uint32_t>(kk & 3) * 32u) >> 4;
+      };
+      if (pc.valid) {
+        // pairs -2 and -1: S_0 and S_1 alone (stages 0 and 1)
+        for (int n = 0; n < 2; ++n) {
+          if (!wait_one(bar(L::kStageFull + n), 0u, ctl, 4)) goto mma_done;
+          if (sc.valid) {
+            if (!wait_q(sc)) goto mma_done;
+            tc_fence_after();
+            const uint64_t qd = qdesc0 + ((static_cast<uint32_t>(sc.qi & 1) * kQTile) >> 4);
+            const uint64_t kd = sdesc_sw128(base + L::kRing + static_cast<uint32_t>(n) * kStage, 16, 1024);
+            const uint32_t d_s = tmem + kColS + 128u * static_cast<uint32_t>(n);
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk)
+              tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
+            if (sc.last_of_item()) tc2_commit_mc(bar(L::kQEmpty + (sc.qi & 1)), 3);
+            sc.advance(args);
+          }
+          tc2_commit_mc(bar(L::kPairDone + 2 + n), 3);
+        }
+        // pairs t >= 0
+        for (;;) {
+          const int t = pc.t;
+          const bool first = pc.j == 0;
+          // P_t ready, which also covers stage t + 2 and the previous item's O reads
+          if (!wait_cl(bar(L::kPFull + (t & 1)), static_cast<uint32_t>(t >> 1) & 1u, ctl, 7)) break;
+          const bool has_s = sc.valid;
+          const int s_qb = sc.qi & 1;
+          const bool s_last = has_s && sc.last_of_item();
+          if (has_s && !wait_q(sc)) break;
+          tc_fence_after();
+          const uint32_t st = base + L::kRing + static_cast<uint32_t>((t + 2) & (kStages - 1)) * kStage;
+          const uint64_t vd = sdesc_sw128(st + kKHalf, kBoxBytes, 1024);
+          const uint32_t a_p = tmem + kColP + 64u * static_cast<uint32_t>(t & 1);
+          if (has_s) {
+            const uint64_t kd = sdesc_sw128(st, 16, 1024);
+            const uint64_t qd = qdesc0 + ((static_cast<uint32_t>(s_qb) * kQTile) >> 4);
+            const uint32_t d_s = tmem + kColS + 128u * static_cast<uint32_t>(t & 1);
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {
+              tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, (first && kk == 0) ? 0u : 1u);
+              tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
+            }
+            if (s_last) tc2_commit_mc(bar(L::kQEmpty + s_qb), 3);
+            sc.advance(args);
+          } else {
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk)
+              tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, (first && kk == 0) ? 0u : 1u);
+          }
+          tc2_commit_mc(bar(L::kPairDone + (t & 3)), 3);
+          pc.advance(args);
+          if (!pc.valid) break;
+        }
+      mma_done:
+        // every MMA of the pair must finish before TMEM is freed
+        tc2_commit_mc(bar(L::kMmaDone), 1);
+        drain_one(bar(L::kMmaDone), 0u, args.timeout_ns);
+      }
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ softmax (both CTAs)
+    const int quarter = warp & 3;
+    const int half = warp >> 2;
+    const int trow = quarter * 32 + lane;              // row within this CTA's 128 rows (= TMEM lane)
+    const int prow = 128 * static_cast<int>(rank) + trow;  // row within the item
+    const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
+    const uint32_t col0 = 64u * static_cast<uint32_t>(half);
+    constexpr int kOCols = D / 2;
+    const float sl2 = args.scale_log2;
+    float* xbuf = reinterpret_cast<float*>(base_ptr + L::kXBuf);
+    const uint32_t xbar = bar(L::kXchg + quarter);
+    uint32_t x_phase = 0;
+    int t = 0;
+    // wait until pair p is complete (both CTAs see the multicast commit)
+    auto wait_pair = [&](int p, int where) -> bool {
+      return wait_cl_warp(bar(L::kPairDone + (p & 3)), pair_parity(p), ctl, where);
+    };
+    auto exchange = [&](float v, float& other, int where) -> bool {
+      float* slot = xbuf + (x_phase & 1u) * 256;
+      slot[half * 128 + trow] = v;
+      mbar_arrive(xbar);
+      if (!wait_warp(xbar, x_phase & 1u, ctl, where)) return false;
+      other = slot[(half ^ 1) * 128 + trow];
+      ++x_phase;
+      return true;
+    };
+    for (int item = cluster; item < args.n_items; item += n_clusters) {
+      Task tk;
+      int head;
+      decode_item(args, item, tk, head);
+      int na;
+      const int nkv = n_key_tiles(tk, na);
+      const bool row_ok = prow < tk.q_rows;
+      const int64_t grow = static_cast<int64_t>(tk.q_row0) + prow;
+      __nv_bfloat16* orow = args.out + grow * args.row_stride + static_cast<int64_t>(head) * D + half * kOCols;
+      if (nkv == 0) {
+        if (row_ok) {
+          uint4 z = make_uint4(0, 0, 0, 0);
+          for (int c = 0; c < kOCols / 8; ++c) reinterpret_cast<uint4*>(orow)[c] = z;
+          if (args.lse && half == 0) args.lse[grow * args.num_heads + head] = -INFINITY;
+        }
+        continue;
+      }
+      float m_run = 0.f, l_run = 0.f;
+      for (int j = 0; j < nkv; ++j, ++t) {
+        const int b = t & 1;
+        const TileSrc src = tile_src(tk, na, j);
+        // S_t is ready and P buffer b is free once pair t - 2 is complete
+        if (!wait_pair(t - 2, 8)) goto softmax_done;
+        tc_fence_after();
+        const uint32_t t_s = tmem + lane_off + kColS + 128u * b + col0;
+        uint32_t r0[32], r1[32];
+        tmem_ld32(t_s + 0u, r0);
+        tmem_ld32(t_s + 32u, r1);
+        tmem_wait_ld(r0);
+        tmem_wait_ld(r1);
+        float s[64];
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          s[c] = __uint_as_float(r0[c]);
+          s[32 + c] = __uint_as_float(r1[c]);
+        }
+        const int valid = src.valid - static_cast<int>(col0);
+        if (valid < 64) {
+#pragma unroll
+          for (int c = 0; c < 64; ++c)
+            if (c >= valid) s[c] = -INFINITY;
+        }
+        float mx[32];
+#pragma unroll
+        for (int c = 0; c < 32; ++c) mx[c] = fmaxf(s[c], s[c + 32]);
+#pragma unroll
+        for (int w = 16; w >= 1; w >>= 1)
+#pragma unroll
+          for (int c = 0; c < w; ++c) mx[c] = fmaxf(mx[c], mx[c + w]);
+        float mo;
+        if (!exchange(mx[0], mo, 11)) goto softmax_done;
+        const float m_tile = fmaxf(mx[0], mo) * sl2;
+        if (j == 0) {
+          m_run = m_tile;
+        } else if (__any_sync(0xffffffffu, m_tile > m_run + 8.0f)) {
+          // O must first hold P_t-1 V_t-1: pair t - 1 complete
+          if (!wait_pair(t - 1, 9)) goto softmax_done;
+          tc_fence_after();
+          const float m_new = fmaxf(m_run, m_tile);
+          const float alpha = ex2_approx(m_run - m_new);
+          m_run = m_new;
+          l_run *= alpha;
+          const uint32_t t_o = tmem + lane_off + kColO + static_cast<uint32_t>(half * kOCols);
+#pragma unroll
+          for (int cc = 0; cc < kOCols / 16; ++cc) {
+            uint32_t o[16];
+            tmem_ld16(t_o + 16u * cc, o);
+            tmem_wait_ld(o);
+#pragma unroll
+            for (int c = 0; c < 16; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * alpha);
+            tmem_st16(t_o + 16u * cc, o);
+          }
+        }
+        const float neg_m = -m_run;
+        const uint32_t t_p = tmem + lane_off + kColP + 64u * b + 32u * static_cast<uint32_t>(half);
+        float ls[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          uint32_t pk[8];
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            const float x = ex2_approx(fmaf(s[16 * q + 2 * c], sl2, neg_m));
+            const float y = ex2_approx(fmaf(s[16 * q + 2 * c + 1], sl2, neg_m));
+            ls[(2 * c) & 3] += x;
+            ls[(2 * c + 1) & 3] += y;
+            pk[c] = pack_bf16x2(x, y);
+          }
+          tmem_st8(t_p + 8u * q, pk);
+        }
+        l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+        // the MMA thread waits only for P: the leader's warp 0 first makes
+        // sure that pair t's ring stage (t + 2) has landed
+        if (leader && warp == 0 &&
+            !wait_warp(bar(L::kStageFull + ((t + 2) & (kStages - 1))), static_cast<uint32_t>((t + 2) / kStages) & 1u,
+                       ctl, 13))
+          goto softmax_done;
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(mapa_shared(bar(L::kPFull + b), 0));
+      }
+      {
+        float l_other;
+        if (!exchange(l_run, l_other, 12)) goto softmax_done;
+        const float l_row = l_run + l_other;
+        if (!wait_pair(t - 1, 10)) goto softmax_done;  // the item's last pair
+        tc_fence_after();
+        const float inv_l = 1.0f / l_row;
+        const uint32_t t_o = tmem + lane_off + kColO + static_cast<uint32_t>(half * kOCols);
+        uint32_t packed[kOCols / 2];
+#pragma unroll
+        for (int cc = 0; cc < kOCols / 32; ++cc) {
+          uint32_t o[32];
+          tmem_ld32(t_o + 32u * cc, o);
+          tmem_wait_ld(o);
+#pragma unroll
+          for (int c = 0; c < 16; ++c)
+            packed[16 * cc + c] =
+                pack_bf16x2(__uint_as_float(o[2 * c]) * inv_l, __uint_as_float(o[2 * c + 1]) * inv_l);
+        }
+        // (the next arrival on p_full, after the next tile's P, tells the MMA
+        // thread that these O reads are done)
+        tc_fence_before();
+        if (row_ok) {
+          uint4* dst = reinterpret_cast<uint4*>(orow);
+#pragma unroll
+          for (int c = 0; c < kOCols / 8; ++c)
+            dst[c] = make_uint4(packed[4 * c], packed[4 * c + 1], packed[4 * c + 2], packed[4 * c + 3]);
+          if (args.lse && half == 0)
+            args.lse[grow * args.num_heads + head] = (m_run + log2f(l_row)) * 0.69314718055994530942f;
+        }
+      }
+    }
+  softmax_done:;
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // the pair's MMAs and TMEM reads are over in both CTAs
+  if (warp == 9) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem, kTmemCols);
+  }
+  cluster_sync();
+}
+
+}  // namespace rc

@@ -1,6 +1,6 @@
 // common.cuh -- work description shared by the attention kernels.
 //
-// One task is a run of at most 128 consecutive query rows that all see the
+// One task is a run of at most 256 consecutive query rows that all see the
 // same keys: a key range A in one K/V pair and an optional key range B in a
 // second K/V pair.  The joint masks of the paper reduce to such tasks
 // (Sec. 3.3, App. C):
@@ -19,7 +19,7 @@ namespace rc {
 
 struct Task {
   int32_t q_row0;  // first query row (row of the Q/O tensors)
-  int32_t q_rows;  // rows in this task, 1..128
+  int32_t q_rows;  // rows in this task, 1..rows_per_task (128 or 256)
   int32_t a_row0;  // key range A: first row in the A tensors
   int32_t a_len;   //              length
   int32_t b_row0;  // key range B (in the B tensors)
@@ -38,7 +38,7 @@ struct AttnArgs {
   float* lse;                   // [rows, H] or null
   int64_t row_stride;           // elements between rows of Q/K/V/O (= H * D)
   float scale_log2;             // softmax_scale * log2(e)
-  uint32_t pad;
+  int32_t rows_per_task;        // 128 or 256 (the mma.sync kernel splits tasks into 64-row CTAs)
   uint64_t timeout_ns;          // bound of every in-kernel wait
   // raw pointers, used by the mma.sync kernel (the tcgen05 kernel reads
   // through tensor maps)

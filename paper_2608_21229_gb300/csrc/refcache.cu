@@ -18,6 +18,7 @@
 #include "refcache.h"
 #include "attn_mma.cuh"
 #include "attn_tc.cuh"
+#include "attn_tc2.cuh"
 
 using rc::AttnArgs;
 using rc::CopySeg;
@@ -50,7 +51,8 @@ struct DeviceInfo {
   bool checked = false;
   bool ok = false;
   int num_sms = 0;
-  bool attr_set[4] = {false, false, false, false};
+  bool attr_set[5] = {false, false, false, false, false};
+  int max_clusters = 0;
 };
 DeviceInfo g_dev[kMaxDevices];
 std::mutex g_dev_mu;
@@ -103,13 +105,13 @@ EncodeTiledFn encode_fn() {
 }
 
 // THD bf16 tensor [rows, H, D] seen as a 2-D array (H*D columns, rows rows);
-// box = 64 columns (128 bytes) x 128 rows with the 128-byte swizzle.
-int make_tmap(CUtensorMap* m, const void* base, int64_t rows, int H, int D) {
+// box = 64 columns (128 bytes) x box_rows rows with the 128-byte swizzle.
+int make_tmap(CUtensorMap* m, const void* base, int64_t rows, int H, int D, uint32_t box_rows = 128) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return fail(REFCACHE_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
   const cuuint64_t dims[2] = {static_cast<cuuint64_t>(H) * D, static_cast<cuuint64_t>(std::max<int64_t>(rows, 1))};
   const cuuint64_t strides[1] = {static_cast<cuuint64_t>(H) * D * 2};
-  const cuuint32_t box[2] = {64, 128};
+  const cuuint32_t box[2] = {64, box_rows};
   const cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -119,13 +121,15 @@ int make_tmap(CUtensorMap* m, const void* base, int64_t rows, int H, int D) {
 }
 
 // ---------------------------------------------------------------- work lists
-constexpr int kTaskRows = 128;  // query rows per task (the tcgen05 kernel's tile)
+// Query rows per task: one M = 256 MMA of a CTA pair for head_dim 128, one
+// 128-row tile of a single CTA for head_dim 64.
+int task_rows(int D) { return D == 128 ? 256 : 128; }
 
-void add_rows(std::vector<Task>& v, int q0, int qn, int a0, int an, int b0, int bn) {
-  for (int r = 0; r < qn; r += kTaskRows) {
+void add_rows(std::vector<Task>& v, int rows_per_task, int q0, int qn, int a0, int an, int b0, int bn) {
+  for (int r = 0; r < qn; r += rows_per_task) {
     Task t{};
     t.q_row0 = q0 + r;
-    t.q_rows = std::min(kTaskRows, qn - r);
+    t.q_rows = std::min(rows_per_task, qn - r);
     t.a_row0 = a0;
     t.a_len = an;
     t.b_row0 = b0;
@@ -186,6 +190,29 @@ int launch_tc(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info,
   return REFCACHE_OK;
 }
 
+// The CTA-pair kernel (head_dim 128): grid = 2 x the clusters that fit at once.
+int launch_tc2(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info, cudaStream_t s) {
+  constexpr uint32_t smem = rc::tc2::Smem::kDynamic;
+  if (!info->attr_set[4]) {
+    cudaError_t e = cudaFuncSetAttribute(rc::attn_tc2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_tc2_kernel)");
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(2 * static_cast<unsigned>(info->num_sms / 2), 1, 1);
+    cfg.blockDim = dim3(rc::tc2::kThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    int clusters = 0;
+    e = cudaOccupancyMaxActiveClusters(&clusters, rc::attn_tc2_kernel, &cfg);
+    if (e != cudaSuccess || clusters < 1) clusters = info->num_sms / 2;
+    info->max_clusters = clusters;
+    info->attr_set[4] = true;
+  }
+  const int clusters = std::min(a.n_items, info->max_clusters);
+  rc::attn_tc2_kernel<<<2 * clusters, rc::tc2::kThreads, smem, s>>>(maps[0], maps[1], maps[2], maps[3], maps[4], a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "attn_tc2_kernel launch");
+  return REFCACHE_OK;
+}
+
 template <int D>
 int launch_mma(const AttnArgs& a, DeviceInfo* info, cudaStream_t s) {
   constexpr int smem = 5 * 64 * D * 2;
@@ -195,7 +222,7 @@ int launch_mma(const AttnArgs& a, DeviceInfo* info, cudaStream_t s) {
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_mma_kernel)");
     info->attr_set[key] = true;
   }
-  rc::attn_mma_kernel<D><<<a.n_items * 2, 128, smem, s>>>(a);
+  rc::attn_mma_kernel<D><<<a.n_items * (a.rows_per_task / 64), 128, smem, s>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "attn_mma_kernel launch");
   return REFCACHE_OK;
@@ -224,6 +251,7 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
   a.lse = op.lse;
   a.row_stride = static_cast<int64_t>(H) * D;
   a.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634074);
+  a.rows_per_task = task_rows(D);
   a.timeout_ns = g_timeout_ns.load();
   a.q = static_cast<const __nv_bfloat16*>(op.q);
   a.ka = static_cast<const __nv_bfloat16*>(op.ka);
@@ -233,20 +261,22 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
   if (static_cast<int64_t>(n_tasks) * H > (1ll << 30)) return fail(REFCACHE_ERR_INVALID_ARG, "too many work items");
   if (g_kernel.load() == REFCACHE_KERNEL_MMA_SYNC)
     return D == 64 ? launch_mma<64>(a, info, s) : launch_mma<128>(a, info, s);
+  // K tiles of the CTA-pair kernel are loaded as two 64-row halves
+  const uint32_t k_rows = D == 128 ? 64 : 128;
   CUtensorMap maps[5];
   int rc;
   if ((rc = make_tmap(&maps[0], op.q, op.q_rows, H, D)) != 0) return rc;
-  if ((rc = make_tmap(&maps[1], op.ka, op.a_rows, H, D)) != 0) return rc;
+  if ((rc = make_tmap(&maps[1], op.ka, op.a_rows, H, D, k_rows)) != 0) return rc;
   if ((rc = make_tmap(&maps[2], op.va, op.a_rows, H, D)) != 0) return rc;
   if (op.kb && op.b_rows > 0) {
-    if ((rc = make_tmap(&maps[3], op.kb, op.b_rows, H, D)) != 0) return rc;
+    if ((rc = make_tmap(&maps[3], op.kb, op.b_rows, H, D, k_rows)) != 0) return rc;
     if ((rc = make_tmap(&maps[4], op.vb, op.b_rows, H, D)) != 0) return rc;
   } else {
     maps[3] = maps[1];
     maps[4] = maps[2];
   }
   a.dbg_skip_first_load = g_dbg_skip.exchange(0);
-  return D == 64 ? launch_tc<64>(maps, a, info, s) : launch_tc<128>(maps, a, info, s);
+  return D == 64 ? launch_tc<64>(maps, a, info, s) : launch_tc2(maps, a, info, s);
 }
 
 // Work list of full_attention_noalloc: a fixed array in static device memory
@@ -317,6 +347,7 @@ int cache_plan(int num_layers, int mode, const refcache_segments_t* seg, refcach
   }
   if (cache_off[B] > max_rows) return fail(REFCACHE_ERR_INVALID_ARG, "cache rows too large");
   const int H = seg->num_heads, D = seg->head_dim;
+  const int tr = task_rows(D);
   std::vector<Task> bt, st;
   std::vector<CopySeg> cp;
   for (int b = 0; b < B; ++b) {
@@ -324,12 +355,12 @@ int cache_plan(int num_layers, int mode, const refcache_segments_t* seg, refcach
     const int l0 = seg->cu_live[b], nl = seg->cu_live[b + 1] - l0;
     const int c0 = static_cast<int>(cache_off[b]), nc = static_cast<int>(cache_off[b + 1] - cache_off[b]);
     if (mode == REFCACHE_MASK_BEYOND_ALT) {
-      add_rows(bt, s0, na, s0, na, 0, 0);            // anchor rows attend anchors only
-      add_rows(bt, s0 + na, ns - na, s0, ns, 0, 0);  // reference rows attend [ST; R]
+      add_rows(bt, tr, s0, na, s0, na, 0, 0);            // anchor rows attend anchors only
+      add_rows(bt, tr, s0 + na, ns - na, s0, ns, 0, 0);  // reference rows attend [ST; R]
     } else {
-      add_rows(bt, s0, ns, s0, ns, 0, 0);  // [ST; R] rows attend [ST; R] (R only when isolated)
+      add_rows(bt, tr, s0, ns, s0, ns, 0, 0);  // [ST; R] rows attend [ST; R] (R only when isolated)
     }
-    add_rows(st, l0, nl, l0, nl, c0, nc);  // live rows attend their own rows, then the cache
+    add_rows(st, tr, l0, nl, l0, nl, c0, nc);  // live rows attend their own rows, then the cache
     if (nc > 0) {
       CopySeg c{};
       c.src_row0 = mode == REFCACHE_MASK_BEYOND_ALT ? s0 : s0 + na;
@@ -552,7 +583,7 @@ int full_attention(int batch, int num_heads, int head_dim, const int32_t* cu_seq
   std::vector<Task> tasks;
   for (int b = 0; b < batch; ++b) {
     const int s0 = cu_seqlens[b], n = cu_seqlens[b + 1] - s0;
-    add_rows(tasks, s0, n, s0, n, 0, 0);
+    add_rows(tasks, task_rows(head_dim), s0, n, s0, n, 0, 0);
   }
   order_tasks(tasks);
   if (tasks.empty()) return REFCACHE_OK;
@@ -588,12 +619,13 @@ int full_attention_noalloc(int batch, int num_heads, int head_dim, const int32_t
   if (rc) return rc;
   if ((rc = check_cu(cu_seqlens, batch, "cu_seqlens", (1ll << 31) - 1 - 512)) != 0) return rc;
   if ((rc = check_scale(softmax_scale)) != 0) return rc;
+  const int tr = task_rows(head_dim);
   int64_t n_tasks = 0;
-  for (int b = 0; b < batch; ++b) n_tasks += (cu_seqlens[b + 1] - cu_seqlens[b] + kTaskRows - 1) / kTaskRows;
+  for (int b = 0; b < batch; ++b) n_tasks += (cu_seqlens[b + 1] - cu_seqlens[b] + tr - 1) / tr;
   if (n_tasks > REFCACHE_NOALLOC_MAX_TASKS)
     return fail(REFCACHE_ERR_INVALID_ARG,
-                "full_attention_noalloc: %lld work items exceed the static limit of %d (128 query rows each)",
-                static_cast<long long>(n_tasks), REFCACHE_NOALLOC_MAX_TASKS);
+                "full_attention_noalloc: %lld work items exceed the static limit of %d (%d query rows each)",
+                static_cast<long long>(n_tasks), REFCACHE_NOALLOC_MAX_TASKS, tr);
   const int64_t rows = cu_seqlens[batch];
   if ((rc = check_ptrs({q, k, v, o}, rows, "full_attention_noalloc")) != 0) return rc;
   DeviceInfo* info = nullptr;
@@ -615,10 +647,10 @@ int full_attention_noalloc(int batch, int num_heads, int head_dim, const int32_t
   int n = 0;
   for (int b = 0; b < batch; ++b) {
     const int s0 = cu_seqlens[b], len = cu_seqlens[b + 1] - s0;
-    for (int r = 0; r < len; r += kTaskRows) {
+    for (int r = 0; r < len; r += tr) {
       Task t{};
       t.q_row0 = s0 + r;
-      t.q_rows = std::min(kTaskRows, len - r);
+      t.q_rows = std::min(tr, len - r);
       t.a_row0 = s0;
       t.a_len = len;
       g_noalloc_host[n++] = t;
