@@ -13,12 +13,15 @@
 // CTA keeps its own 128 query rows (A is split along M).  Per SM this halves
 // the tile bytes fetched and the B-operand bytes read, for the same MMA work.
 //
-// Cluster of 2 CTAs (rank 0 = leader), 320 threads each:
-//   warps 0-7  softmax of this CTA's 128 rows (as in attn_tc.cuh)
-//   warp 8     TMA producer: this CTA's Q rows and its halves of the K and V
+// Cluster of 2 CTAs (rank 0 = leader), 192 threads each:
+//   warps 0-3  softmax: thread l of warp w owns row 32 w + l of this CTA's
+//              128 rows (its TMEM lane), all 128 score columns of a tile
+//   warp 4     TMA producer: this CTA's Q rows and its halves of the K and V
 //              tiles; completion is counted on the leader's barriers
-//   warp 9     both CTAs: TMEM allocation (a pair operation); leader only:
+//   warp 5     both CTAs: TMEM allocation (a pair operation); leader only:
 //              the MMA thread
+// One softmax warp per SM sub-partition leaves the MMA warp's sub-partition
+// with a single busy warp beside it, and a row needs no partner thread.
 // An item is a task of up to 256 query rows: CTA r takes rows
 // [128 r, 128 r + 128).  Items are taken cluster by cluster, head-major.
 //
@@ -52,14 +55,15 @@ namespace rc {
 namespace tc2 {
 using tc::Ctl;
 constexpr int kD = 128;
-constexpr int kThreads = 320;
+constexpr int kThreads = 192;
 constexpr int kStages = 4;                  // ring stages (pair_done has as many barriers)
 constexpr uint32_t kKHalf = 64 * 128 * 2;   // 16 KB: this CTA's 64 keys x 128 d of a K tile
 constexpr uint32_t kVHalf = 128 * 64 * 2;   // 16 KB: 128 keys x this CTA's 64 d of a V tile
 constexpr uint32_t kStage = kKHalf + kVHalf;
 constexpr uint32_t kQTile = 128 * 128 * 2;
 constexpr uint32_t kKBox = 64 * 128;        // one K box: 64 rows x 128 bytes
-constexpr int kWarpArrivals = 16;           // 8 softmax warps in each of the 2 CTAs
+constexpr int kWarpArrivals = 8;            // 4 softmax warps in each of the 2 CTAs
+constexpr int kProducerWarp = 4, kMmaWarp = 5;
 static_assert(kStages == 4, "pair_done indexing assumes four stages");
 
 struct Smem {
@@ -67,9 +71,8 @@ struct Smem {
   static constexpr uint32_t kRing = 2 * kQTile;    // stage s: [K half | V half]
   static constexpr uint32_t kBars = kRing + kStages * kStage;
   static constexpr int kQFull = 0, kQEmpty = 2, kStageFull = 4, kPairDone = 4 + kStages, kPFull = kPairDone + 4,
-                       kMmaDone = kPFull + 2, kXchg = kMmaDone + 1, kNumBars = kXchg + 4;
-  static constexpr uint32_t kXBuf = kBars + 8 * kNumBars;
-  static constexpr uint32_t kTmemHolder = kXBuf + 2 * 2 * 128 * 4;
+                       kMmaDone = kPFull + 2, kNumBars = kMmaDone + 1;
+  static constexpr uint32_t kTmemHolder = kBars + 8 * kNumBars;
   static constexpr uint32_t kAbort = kTmemHolder + 4;
   static constexpr uint32_t kUsed = kAbort + 4;
   static constexpr uint32_t kMaxDynamic = 232448;
@@ -152,12 +155,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
       mbar_init(bar(L::kPairDone + s), 1);
     }
     mbar_init(bar(L::kMmaDone), 1);
-    for (int q = 0; q < 4; ++q) mbar_init(bar(L::kXchg + q), 64);
     *abort_flag = 0;
     fence_barrier_init();
     fence_proxy_async_smem();
   }
-  if (warp == 9) {
+  if (warp == tc2::kMmaWarp) {
     tmem_alloc_pair(smem_u32(tmem_holder), kTmemCols);
     tmem_relinquish_pair();
   }
@@ -169,7 +171,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
   const Ctl ctl{abort_flag, args.timeout_ns};
   auto lbar = [&](int i) -> uint32_t { return mapa_shared(bar(i), 0); };  // leader's barrier i
 
-  if (warp == 8) {
+  if (warp == tc2::kProducerWarp) {
     // ------------------------------------------------------------ producer (both CTAs)
     // Stages u = 0 .. T+1 in order: K_u (u < T) and V_u-2 (u >= 2), this
     // CTA's halves.  Stage 1 of a one-tile stream is empty.  An item's Q rows
@@ -253,7 +255,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         if (q_armed[b] >= 0) drain_one(bar(L::kQFull + b), static_cast<uint32_t>(q_armed[b]) & 1u, args.timeout_ns);
     }
     __syncwarp();
-  } else if (warp == 9) {
+  } else if (warp == tc2::kMmaWarp) {
     // ------------------------------------------------------------ MMA issuer (leader)
     if (leader && lane == 0) {
       Cursor sc, pc;  // S side (two tiles ahead) and P.V side of the stream
@@ -332,30 +334,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
     __syncwarp();
   } else {
     // ------------------------------------------------------------ softmax (both CTAs)
-    const int quarter = warp & 3;
-    const int half = warp >> 2;
-    const int trow = quarter * 32 + lane;              // row within this CTA's 128 rows (= TMEM lane)
+    const int trow = warp * 32 + lane;                     // row within this CTA's 128 rows (= TMEM lane)
     const int prow = 128 * static_cast<int>(rank) + trow;  // row within the item
-    const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
-    const uint32_t col0 = 64u * static_cast<uint32_t>(half);
-    constexpr int kOCols = D / 2;
+    const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
     const float sl2 = args.scale_log2;
-    float* xbuf = reinterpret_cast<float*>(base_ptr + L::kXBuf);
-    const uint32_t xbar = bar(L::kXchg + quarter);
-    uint32_t x_phase = 0;
+    const f32x2 sl2x2 = make_f32x2(sl2, sl2);
     int t = 0;
     // wait until pair p is complete (both CTAs see the multicast commit)
     auto wait_pair = [&](int p, int where) -> bool {
       return wait_cl_warp(bar(L::kPairDone + (p & 3)), pair_parity(p), ctl, where);
-    };
-    auto exchange = [&](float v, float& other, int where) -> bool {
-      float* slot = xbuf + (x_phase & 1u) * 256;
-      slot[half * 128 + trow] = v;
-      mbar_arrive(xbar);
-      if (!wait_warp(xbar, x_phase & 1u, ctl, where)) return false;
-      other = slot[(half ^ 1) * 128 + trow];
-      ++x_phase;
-      return true;
     };
     for (int item = cluster; item < args.n_items; item += n_clusters) {
       Task tk;
@@ -365,12 +352,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
       const int nkv = n_key_tiles(tk, na);
       const bool row_ok = prow < tk.q_rows;
       const int64_t grow = static_cast<int64_t>(tk.q_row0) + prow;
-      __nv_bfloat16* orow = args.out + grow * args.row_stride + static_cast<int64_t>(head) * D + half * kOCols;
+      __nv_bfloat16* orow = args.out + grow * args.row_stride + static_cast<int64_t>(head) * D;
       if (nkv == 0) {
         if (row_ok) {
           uint4 z = make_uint4(0, 0, 0, 0);
-          for (int c = 0; c < kOCols / 8; ++c) reinterpret_cast<uint4*>(orow)[c] = z;
-          if (args.lse && half == 0) args.lse[grow * args.num_heads + head] = -INFINITY;
+          for (int c = 0; c < D / 8; ++c) reinterpret_cast<uint4*>(orow)[c] = z;
+          if (args.lse) args.lse[grow * args.num_heads + head] = -INFINITY;
         }
         continue;
       }
@@ -381,34 +368,41 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         // S_t is ready and P buffer b is free once pair t - 2 is complete
         if (!wait_pair(t - 2, 8)) goto softmax_done;
         tc_fence_after();
-        const uint32_t t_s = tmem + lane_off + kColS + 128u * b + col0;
-        uint32_t r0[32], r1[32];
-        tmem_ld32(t_s + 0u, r0);
-        tmem_ld32(t_s + 32u, r1);
-        tmem_wait_ld(r0);
-        tmem_wait_ld(r1);
-        float s[64];
+        const uint32_t t_s = tmem + lane_off + kColS + 128u * b;
+        float s[128];
+        {
+          uint32_t r0[32], r1[32], r2[32], r3[32];
+          tmem_ld32(t_s + 0u, r0);
+          tmem_ld32(t_s + 32u, r1);
+          tmem_ld32(t_s + 64u, r2);
+          tmem_ld32(t_s + 96u, r3);
+          tmem_wait_ld(r0);
+          tmem_wait_ld(r1);
+          tmem_wait_ld(r2);
+          tmem_wait_ld(r3);
 #pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          s[c] = __uint_as_float(r0[c]);
-          s[32 + c] = __uint_as_float(r1[c]);
+          for (int c = 0; c < 32; ++c) {
+            s[c] = __uint_as_float(r0[c]);
+            s[32 + c] = __uint_as_float(r1[c]);
+            s[64 + c] = __uint_as_float(r2[c]);
+            s[96 + c] = __uint_as_float(r3[c]);
+          }
         }
-        const int valid = src.valid - static_cast<int>(col0);
-        if (valid < 64) {
+        if (src.valid < 128) {  // keys past the end of the range
 #pragma unroll
-          for (int c = 0; c < 64; ++c)
-            if (c >= valid) s[c] = -INFINITY;
+          for (int c = 0; c < 128; ++c)
+            if (c >= src.valid) s[c] = -INFINITY;
         }
-        float mx[32];
+        // row maximum: four independent chains of 3-input max
+        float mx[4];
 #pragma unroll
-        for (int c = 0; c < 32; ++c) mx[c] = fmaxf(s[c], s[c + 32]);
+        for (int k = 0; k < 4; ++k) {
+          mx[k] = fmax3(s[32 * k], s[32 * k + 1], s[32 * k + 2]);
 #pragma unroll
-        for (int w = 16; w >= 1; w >>= 1)
-#pragma unroll
-          for (int c = 0; c < w; ++c) mx[c] = fmaxf(mx[c], mx[c + w]);
-        float mo;
-        if (!exchange(mx[0], mo, 11)) goto softmax_done;
-        const float m_tile = fmaxf(mx[0], mo) * sl2;
+          for (int c = 3; c < 31; c += 2) mx[k] = fmax3(mx[k], s[32 * k + c], s[32 * k + c + 1]);
+          mx[k] = fmaxf(mx[k], s[32 * k + 31]);
+        }
+        const float m_tile = fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3])) * sl2;
         if (j == 0) {
           m_run = m_tile;
         } else if (__any_sync(0xffffffffu, m_tile > m_run + 8.0f)) {
@@ -417,36 +411,52 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
           tc_fence_after();
           const float m_new = fmaxf(m_run, m_tile);
           const float alpha = ex2_approx(m_run - m_new);
+          const f32x2 alpha2 = make_f32x2(alpha, alpha);
           m_run = m_new;
           l_run *= alpha;
-          const uint32_t t_o = tmem + lane_off + kColO + static_cast<uint32_t>(half * kOCols);
+          const uint32_t t_o = tmem + lane_off + kColO;
 #pragma unroll
-          for (int cc = 0; cc < kOCols / 16; ++cc) {
+          for (int cc = 0; cc < D / 16; ++cc) {
             uint32_t o[16];
             tmem_ld16(t_o + 16u * cc, o);
             tmem_wait_ld(o);
 #pragma unroll
-            for (int c = 0; c < 16; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * alpha);
+            for (int c = 0; c < 16; c += 2) {
+              f32x2 v = mul_f32x2(make_f32x2(__uint_as_float(o[c]), __uint_as_float(o[c + 1])), alpha2);
+              float lo, hi;
+              split_f32x2(v, lo, hi);
+              o[c] = __float_as_uint(lo);
+              o[c + 1] = __float_as_uint(hi);
+            }
             tmem_st16(t_o + 16u * cc, o);
           }
         }
-        const float neg_m = -m_run;
-        const uint32_t t_p = tmem + lane_off + kColP + 64u * b + 32u * static_cast<uint32_t>(half);
-        float ls[4] = {0.f, 0.f, 0.f, 0.f};
+        // P = exp2(scale * S - m) as bf16 pairs into P buffer b, 32 keys (16 columns) at a time
+        const f32x2 negm = make_f32x2(-m_run, -m_run);
+        const uint32_t t_p = tmem + lane_off + kColP + 64u * b;
+        f32x2 lacc[4];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          uint32_t pk[8];
+        for (int i = 0; i < 4; ++i) lacc[i] = make_f32x2(0.f, 0.f);
 #pragma unroll
-          for (int c = 0; c < 8; ++c) {
-            const float x = ex2_approx(fmaf(s[16 * q + 2 * c], sl2, neg_m));
-            const float y = ex2_approx(fmaf(s[16 * q + 2 * c + 1], sl2, neg_m));
-            ls[(2 * c) & 3] += x;
-            ls[(2 * c + 1) & 3] += y;
+        for (int k = 0; k < 4; ++k) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int c = 0; c < 16; ++c) {
+            const f32x2 e = fma_f32x2(make_f32x2(s[32 * k + 2 * c], s[32 * k + 2 * c + 1]), sl2x2, negm);
+            float e0, e1;
+            split_f32x2(e, e0, e1);
+            const float x = ex2_approx(e0), y = ex2_approx(e1);
+            lacc[c & 3] = add_f32x2(lacc[c & 3], make_f32x2(x, y));
             pk[c] = pack_bf16x2(x, y);
           }
-          tmem_st8(t_p + 8u * q, pk);
+          tmem_st16(t_p + 16u * k, pk);
         }
-        l_run += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+        {
+          const f32x2 l2 = add_f32x2(add_f32x2(lacc[0], lacc[1]), add_f32x2(lacc[2], lacc[3]));
+          float lo, hi;
+          split_f32x2(l2, lo, hi);
+          l_run += lo + hi;
+        }
         // the MMA thread waits only for P: the leader's warp 0 first makes
         // sure that pair t's ring stage (t + 2) has landed
         if (leader && warp == 0 &&
@@ -459,16 +469,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         if (lane == 0) mbar_arrive_cluster(mapa_shared(bar(L::kPFull + b), 0));
       }
       {
-        float l_other;
-        if (!exchange(l_run, l_other, 12)) goto softmax_done;
-        const float l_row = l_run + l_other;
         if (!wait_pair(t - 1, 10)) goto softmax_done;  // the item's last pair
         tc_fence_after();
-        const float inv_l = 1.0f / l_row;
-        const uint32_t t_o = tmem + lane_off + kColO + static_cast<uint32_t>(half * kOCols);
-        uint32_t packed[kOCols / 2];
+        const float inv_l = 1.0f / l_run;
+        const uint32_t t_o = tmem + lane_off + kColO;
+        uint32_t packed[D / 2];
 #pragma unroll
-        for (int cc = 0; cc < kOCols / 32; ++cc) {
+        for (int cc = 0; cc < D / 32; ++cc) {
           uint32_t o[32];
           tmem_ld32(t_o + 32u * cc, o);
           tmem_wait_ld(o);
@@ -483,10 +490,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         if (row_ok) {
           uint4* dst = reinterpret_cast<uint4*>(orow);
 #pragma unroll
-          for (int c = 0; c < kOCols / 8; ++c)
+          for (int c = 0; c < D / 8; ++c)
             dst[c] = make_uint4(packed[4 * c], packed[4 * c + 1], packed[4 * c + 2], packed[4 * c + 3]);
-          if (args.lse && half == 0)
-            args.lse[grow * args.num_heads + head] = (m_run + log2f(l_row)) * 0.69314718055994530942f;
+          if (args.lse) args.lse[grow * args.num_heads + head] = (m_run + log2f(l_run)) * 0.69314718055994530942f;
         }
       }
     }
@@ -496,7 +502,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
   tc_fence_before();
   __syncthreads();
   cluster_sync();  // the pair's MMAs and TMEM reads are over in both CTAs
-  if (warp == 9) {
+  if (warp == tc2::kMmaWarp) {
     tc_fence_after();
     tmem_dealloc_pair(tmem, kTmemCols);
   }
