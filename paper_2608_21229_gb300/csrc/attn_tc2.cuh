@@ -25,26 +25,31 @@
 // An item is a task of up to 256 query rows: CTA r takes rows
 // [128 r, 128 r + 128).  Items are taken cluster by cluster, head-major.
 //
-// The key tiles of all items a cluster runs form one stream t = 0 .. T-1.
-// Pair p of MMAs (p = -2, -1: S_0, S_1 alone; p >= 0: O += P_p V_p
-// interleaved, MMA by MMA, with S_p+2 = Q K_p+2^T) reads ring stage u = p + 2,
-// which holds K_u (if u < T) and V_u-2 (if u >= 2); the ring has kStages
-// stages of 32 KB per CTA.
+// Work is done item by item (an item = a task of up to 256 rows x one
+// head).  An item with n key tiles is a sequence of n + 2 MMA groups:
+//   group G + 0, G + 1     S_0 = Q K_0^T, S_1 = Q K_1^T (the second is empty
+//                          when n = 1)
+//   group G + 2 + j        O += P_j V_j, interleaved MMA by MMA with
+//                          S_j+2 = Q K_j+2^T when j + 2 < n
+// numbered g = 0, 1, 2, ... over all items of the cluster.  Group g reads
+// ring stage g % 4 (K of its S, V of its P.V; 32 KB per CTA).  Tiles are also
+// numbered over all items (t); S_t and P_t live in TMEM buffer t % 2.
 //
 // Synchronisation is built so that the MMA thread does as little as possible
-// between its MMAs: a tcgen05.mma blocks its thread for about as long as the
-// tensor core takes to run it, and the tensor core queues only a few, so any
-// wait or commit between two MMAs idles the tensor core unless it is short.
-// Per pair the MMA thread waits once (P ready) and commits once:
-//   pair_done[p & 3]   one commit per pair (multicast to both CTAs).  Pair p
-//                      complete means: S_p+2 is in S buffer p % 2, O holds
-//                      P_p V_p, P buffer p % 2 and ring stage p + 2 are free.
-//                      Four barriers, so that no waiter can miss a phase: a
-//                      waiter for pair p holds up pair p + 4.
+// between its MMAs: a tcgen05.mma blocks its thread until the tensor core
+// takes it, and the tensor core queues almost nothing, so every cycle the
+// MMA thread spends between two groups idles the tensor core.  Per group the
+// MMA thread waits once (P ready) and commits once:
+//   pair_done[g % 4]   one commit per group (multicast to both CTAs): its S
+//                      is in TMEM, its P.V is in O, its stage and the P
+//                      buffer it read are free.  Four barriers, so that no
+//                      waiter can miss a phase: a waiter for group g holds up
+//                      group g + 4.
 //   p_full[t % 2]      one arrival per softmax warp of both CTAs.  Its phase
 //                      for tile t means P_t is in TMEM, every softmax thread
 //                      has finished reading O for the previous item, and (the
-//                      leader's warp 0 waited for it) stage t + 2 is full.
+//                      leader's warp 0 waited for it) the stage of P_t V_t's
+//                      group is full.
 //   stage_full[s]      the producers' TMA bytes of both CTAs (leader's barrier)
 //   q_full / q_empty   per Q buffer, once per item
 #pragma once
@@ -80,8 +85,8 @@ struct Smem {
   static_assert(kUsed <= kMaxDynamic, "shared-memory layout too large");
 };
 
-// Phase parity of pair_done[p & 3] that completes with pair p (p >= -2).
-__device__ __forceinline__ uint32_t pair_parity(int p) { return static_cast<uint32_t>((p + 2) >> 2) & 1u; }
+// Phase parity of pair_done[g % 4] / stage_full[g % 4] for group g.
+__device__ __forceinline__ uint32_t group_parity(int g) { return static_cast<uint32_t>(g >> 2) & 1u; }
 
 // Bounded wait with cluster-scope acquire (barriers other CTAs arrive on).
 __device__ __forceinline__ bool wait_cl(uint32_t bar, uint32_t parity, const Ctl& c, int where) {
@@ -116,7 +121,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
   using tc2::kStages;
   using tc2::kVHalf;
   using tc2::kWarpArrivals;
-  using tc2::pair_parity;
+  using tc2::group_parity;
   using tc2::wait_cl;
   using tc2::wait_cl_warp;
   using L = tc2::Smem;
@@ -173,77 +178,68 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
 
   if (warp == tc2::kProducerWarp) {
     // ------------------------------------------------------------ producer (both CTAs)
-    // Stages u = 0 .. T+1 in order: K_u (u < T) and V_u-2 (u >= 2), this
-    // CTA's halves.  Stage 1 of a one-tile stream is empty.  An item's Q rows
-    // go out just before the stage that holds the item's first K tile.
+    // This CTA's halves of the stages of every group, in group order, and an
+    // item's Q rows just before its first stage.
     if (lane == 0) {
       int armed_phase[kStages];
       for (int s = 0; s < kStages; ++s) armed_phase[s] = -1;
       int q_armed[2] = {-1, -1};
       bool skip_next = leader && args.dbg_skip_first_load != 0;
-      Cursor kc, vc;
-      kc.init(args, cluster, n_clusters);
-      vc.init(args, cluster, n_clusters);
-      int u = 0;
-      auto load_q = [&]() -> bool {  // this CTA's 128 query rows of kc's item into Q buffer qi % 2
-        const int b = kc.qi & 1;
-        const uint32_t n = static_cast<uint32_t>(kc.qi >> 1);
-        if (!wait_one(bar(L::kQEmpty + b), (n & 1u) ^ 1u, ctl, 1)) return false;
-        if (leader) {
-          mbar_arrive_expect_tx(bar(L::kQFull + b), 2 * kQTile);
-          q_armed[b] = static_cast<int>(n);
-        }
-        const uint32_t qfull = lbar(L::kQFull + b);
-        for (int ch = 0; ch < 2; ++ch)
-          tma_load_2d_pair(base + L::kQ + b * kQTile + ch * kBoxBytes, &tm_q, qfull, kc.head * D + ch * 64,
-                           kc.task.q_row0 + 128 * static_cast<int>(rank));
-        return true;
-      };
-      // stage u: V of vc's tile (if with_v) and K of kc's tile (if with_k)
-      auto load_stage = [&](bool with_v, bool with_k) -> bool {
-        if (with_k && kc.j == 0 && !load_q()) return false;
-        const int slot = u & (kStages - 1);
-        // the stage's previous use (u - kStages) is read by pair u - kStages - 2
-        if (u >= kStages && !wait_one(bar(L::kPairDone + ((u + 2) & 3)), pair_parity(u - kStages - 2), ctl, 2))
-          return false;
+      int g = 0, qi = 0;
+      Task tk;
+      int head = 0, na = 0;
+      // stage of group g: K tile kj (if kj >= 0) and V tile vj (if vj >= 0) of the item
+      auto load_stage = [&](int kj, int vj) -> bool {
+        const int slot = g & (kStages - 1);
+        // the stage's previous group (g - kStages) must be complete
+        if (g >= kStages && !wait_one(bar(L::kPairDone + slot), group_parity(g - kStages), ctl, 2)) return false;
         const uint32_t dst = base + L::kRing + static_cast<uint32_t>(slot) * kStage;
         const uint32_t full = lbar(L::kStageFull + slot);
-        const uint32_t bytes = 2 * ((with_k ? kKHalf : 0u) + (with_v ? kVHalf : 0u));
+        const uint32_t bytes = 2 * ((kj >= 0 ? kKHalf : 0u) + (vj >= 0 ? kVHalf : 0u));
         if (skip_next) {  // fault injection: the leader never arms or loads this stage
           skip_next = false;
         } else {
           if (leader) {
             mbar_arrive_expect_tx(bar(L::kStageFull + slot), bytes);
-            armed_phase[slot] = (u / kStages) & 1;
+            armed_phase[slot] = static_cast<int>(group_parity(g));
           }
-          if (with_k) {  // keys [64 r, 64 r + 64) of the tile, both head-dim boxes
-            const TileSrc src = tile_src(kc.task, kc.na, kc.j);
+          if (kj >= 0) {  // keys [64 r, 64 r + 64) of the tile, both head-dim boxes
+            const TileSrc src = tile_src(tk, na, kj);
             const void* map = src.in_b ? &tm_kb : &tm_ka;
             for (int ch = 0; ch < 2; ++ch)
-              tma_load_2d_pair(dst + ch * kKBox, map, full, kc.head * D + ch * 64,
-                               src.row + 64 * static_cast<int>(rank));
+              tma_load_2d_pair(dst + ch * kKBox, map, full, head * D + ch * 64, src.row + 64 * static_cast<int>(rank));
           }
-          if (with_v) {  // head-dim columns [64 r, 64 r + 64) of all 128 keys
-            const TileSrc src = tile_src(vc.task, vc.na, vc.j);
+          if (vj >= 0) {  // head-dim columns [64 r, 64 r + 64) of all 128 keys
+            const TileSrc src = tile_src(tk, na, vj);
             const void* map = src.in_b ? &tm_vb : &tm_va;
-            tma_load_2d_pair(dst + kKHalf, map, full, vc.head * D + 64 * static_cast<int>(rank), src.row);
+            tma_load_2d_pair(dst + kKHalf, map, full, head * D + 64 * static_cast<int>(rank), src.row);
           }
         }
-        ++u;
+        ++g;
         return true;
       };
-      if (kc.valid) {
-        for (int n = 0; n < 2; ++n) {
-          const bool with_k = kc.valid;
-          if (!load_stage(false, with_k)) goto producer_done;
-          if (with_k) kc.advance(args);
+      for (int item = cluster; item < args.n_items; item += n_clusters) {
+        decode_item(args, item, tk, head);
+        const int nkv = n_key_tiles(tk, na);
+        if (nkv == 0) continue;
+        {  // this CTA's 128 query rows into Q buffer qi % 2
+          const int b = qi & 1;
+          const uint32_t n = static_cast<uint32_t>(qi >> 1);
+          if (!wait_one(bar(L::kQEmpty + b), (n & 1u) ^ 1u, ctl, 1)) goto producer_done;
+          if (leader) {
+            mbar_arrive_expect_tx(bar(L::kQFull + b), 2 * kQTile);
+            q_armed[b] = static_cast<int>(n);
+          }
+          const uint32_t qfull = lbar(L::kQFull + b);
+          for (int ch = 0; ch < 2; ++ch)
+            tma_load_2d_pair(base + L::kQ + b * kQTile + ch * kBoxBytes, &tm_q, qfull, head * D + ch * 64,
+                             tk.q_row0 + 128 * static_cast<int>(rank));
         }
-        while (vc.valid) {
-          const bool with_k = kc.valid;
-          if (!load_stage(true, with_k)) goto producer_done;
-          vc.advance(args);
-          if (with_k) kc.advance(args);
-        }
+        if (!load_stage(0, -1)) goto producer_done;
+        if (!load_stage(nkv > 1 ? 1 : -1, -1)) goto producer_done;
+        for (int j = 0; j < nkv; ++j)
+          if (!load_stage(j + 2 < nkv ? j + 2 : -1, j)) goto producer_done;
+        ++qi;
       }
     producer_done:
       // the leader's full barriers count both CTAs' bytes: once they complete,
@@ -258,14 +254,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
   } else if (warp == tc2::kMmaWarp) {
     // ------------------------------------------------------------ MMA issuer (leader)
     if (leader && lane == 0) {
-      Cursor sc, pc;  // S side (two tiles ahead) and P.V side of the stream
-      sc.init(args, cluster, n_clusters);
-      pc.init(args, cluster, n_clusters);
+      // descriptors of stage 0 (stage s: + s * kStage / 16) and of Q buffer 0
+      const uint64_t kd0 = sdesc_sw128(base + L::kRing, 16, 1024);
+      const uint64_t vd0 = sdesc_sw128(base + L::kRing + kKHalf, kBoxBytes, 1024);
       const uint64_t qdesc0 = sdesc_sw128(base + L::kQ, 16, 1024);
-      auto wait_q = [&](const Cursor& c) -> bool {
-        if (c.j != 0) return true;
-        return wait_one(bar(L::kQFull + (c.qi & 1)), static_cast<uint32_t>(c.qi >> 1) & 1u, ctl, 3);
-      };
       // S step kk: A = Q (128-row boxes of 16 KB), B = this CTA's 64 keys (64-row boxes of 8 KB)
       auto q_off = [](int kk) -> uint64_t {
         return (static_cast<uint32_t>(kk >> 2) * kBoxBytes + static_cast<uint32_t>(kk & 3) * 32u) >> 4;
@@ -273,60 +265,64 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
       auto k_off = [](int kk) -> uint64_t {
         return (static_cast<uint32_t>(kk >> 2) * kKBox + static_cast<uint32_t>(kk & 3) * 32u) >> 4;
       };
-      if (pc.valid) {
-        // pairs -2 and -1: S_0 and S_1 alone (stages 0 and 1)
-        for (int n = 0; n < 2; ++n) {
-          if (!wait_one(bar(L::kStageFull + n), 0u, ctl, 4)) goto mma_done;
-          if (sc.valid) {
-            if (!wait_q(sc)) goto mma_done;
+      bool issued = false;
+      int g = 0, t0 = 0, qi = 0;
+      for (int item = cluster; item < args.n_items; item += n_clusters) {
+        Task tk;
+        int head, na;
+        decode_item(args, item, tk, head);
+        const int nkv = n_key_tiles(tk, na);
+        if (nkv == 0) continue;
+        const int qb = qi & 1;
+        if (!wait_one(bar(L::kQFull + qb), static_cast<uint32_t>(qi >> 1) & 1u, ctl, 3)) goto mma_done;
+        const uint64_t qd = qdesc0 + ((static_cast<uint32_t>(qb) * kQTile) >> 4);
+        // groups G, G + 1: S_0, S_1
+        for (int n = 0; n < 2; ++n, ++g) {
+          const int slot = g & (kStages - 1);
+          if (!wait_one(bar(L::kStageFull + slot), group_parity(g), ctl, 4)) goto mma_done;
+          if (n < nkv) {
             tc_fence_after();
-            const uint64_t qd = qdesc0 + ((static_cast<uint32_t>(sc.qi & 1) * kQTile) >> 4);
-            const uint64_t kd = sdesc_sw128(base + L::kRing + static_cast<uint32_t>(n) * kStage, 16, 1024);
-            const uint32_t d_s = tmem + kColS + 128u * static_cast<uint32_t>(n);
+            const uint64_t kd = kd0 + static_cast<uint64_t>(slot) * (kStage >> 4);
+            const uint32_t d_s = tmem + kColS + (static_cast<uint32_t>((t0 + n) & 1) << 7);
 #pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk)
-              tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
-            if (sc.last_of_item()) tc2_commit_mc(bar(L::kQEmpty + (sc.qi & 1)), 3);
-            sc.advance(args);
+            for (int kk = 0; kk < D / 16; ++kk) tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
+            issued = true;
+            if (n == nkv - 1) tc2_commit_mc(bar(L::kQEmpty + qb), 3);
           }
-          tc2_commit_mc(bar(L::kPairDone + 2 + n), 3);
+          tc2_commit_mc(bar(L::kPairDone + slot), 3);
         }
-        // pairs t >= 0
-        for (;;) {
-          const int t = pc.t;
-          const bool first = pc.j == 0;
-          // P_t ready, which also covers stage t + 2 and the previous item's O reads
-          if (!wait_cl(bar(L::kPFull + (t & 1)), static_cast<uint32_t>(t >> 1) & 1u, ctl, 7)) break;
-          const bool has_s = sc.valid;
-          const int s_qb = sc.qi & 1;
-          const bool s_last = has_s && sc.last_of_item();
-          if (has_s && !wait_q(sc)) break;
+        // groups G + 2 + j: P_j V_j (+ S_j+2)
+        for (int j = 0; j < nkv; ++j, ++g) {
+          const int t = t0 + j;
+          // P_t ready: also covers this group's stage and the previous item's O reads
+          if (!wait_cl(bar(L::kPFull + (t & 1)), static_cast<uint32_t>(t >> 1) & 1u, ctl, 7)) goto mma_done;
           tc_fence_after();
-          const uint32_t st = base + L::kRing + static_cast<uint32_t>((t + 2) & (kStages - 1)) * kStage;
-          const uint64_t vd = sdesc_sw128(st + kKHalf, kBoxBytes, 1024);
-          const uint32_t a_p = tmem + kColP + 64u * static_cast<uint32_t>(t & 1);
-          if (has_s) {
-            const uint64_t kd = sdesc_sw128(st, 16, 1024);
-            const uint64_t qd = qdesc0 + ((static_cast<uint32_t>(s_qb) * kQTile) >> 4);
-            const uint32_t d_s = tmem + kColS + 128u * static_cast<uint32_t>(t & 1);
+          const int slot = g & (kStages - 1);
+          const uint64_t soff = static_cast<uint64_t>(slot) * (kStage >> 4);
+          const uint64_t vd = vd0 + soff;
+          const uint32_t a_p = tmem + kColP + (static_cast<uint32_t>(t & 1) << 6);
+          const uint32_t acc0 = j > 0 ? 1u : 0u;
+          if (j + 2 < nkv) {
+            const uint64_t kd = kd0 + soff;
+            const uint32_t d_s = tmem + kColS + (static_cast<uint32_t>(t & 1) << 7);
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk) {
-              tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, (first && kk == 0) ? 0u : 1u);
+              tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, kk > 0 ? 1u : acc0);
               tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
             }
-            if (s_last) tc2_commit_mc(bar(L::kQEmpty + s_qb), 3);
-            sc.advance(args);
+            if (j + 2 == nkv - 1) tc2_commit_mc(bar(L::kQEmpty + qb), 3);
           } else {
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk)
-              tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, (first && kk == 0) ? 0u : 1u);
+              tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, kk > 0 ? 1u : acc0);
           }
-          tc2_commit_mc(bar(L::kPairDone + (t & 3)), 3);
-          pc.advance(args);
-          if (!pc.valid) break;
+          tc2_commit_mc(bar(L::kPairDone + slot), 3);
         }
-      mma_done:
-        // every MMA of the pair must finish before TMEM is freed
+        t0 += nkv;
+        ++qi;
+      }
+    mma_done:
+      if (issued) {  // every MMA must finish before TMEM is freed
         tc2_commit_mc(bar(L::kMmaDone), 1);
         drain_one(bar(L::kMmaDone), 0u, args.timeout_ns);
       }
@@ -339,10 +335,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
     const float sl2 = args.scale_log2;
     const f32x2 sl2x2 = make_f32x2(sl2, sl2);
-    int t = 0;
-    // wait until pair p is complete (both CTAs see the multicast commit)
-    auto wait_pair = [&](int p, int where) -> bool {
-      return wait_cl_warp(bar(L::kPairDone + (p & 3)), pair_parity(p), ctl, where);
+    int t = 0;  // tiles of earlier items
+    int G = 0;  // first group of the item
+    // wait until group g is complete (both CTAs see the multicast commit)
+    auto wait_group = [&](int g, int where) -> bool {
+      return wait_cl_warp(bar(L::kPairDone + (g & 3)), group_parity(g), ctl, where);
     };
     for (int item = cluster; item < args.n_items; item += n_clusters) {
       Task tk;
@@ -365,8 +362,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
       for (int j = 0; j < nkv; ++j, ++t) {
         const int b = t & 1;
         const TileSrc src = tile_src(tk, na, j);
-        // S_t is ready and P buffer b is free once pair t - 2 is complete
-        if (!wait_pair(t - 2, 8)) goto softmax_done;
+        // S_j is ready and P buffer b is free once group G + j is complete
+        if (!wait_group(G + j, 8)) goto softmax_done;
         tc_fence_after();
         const uint32_t t_s = tmem + lane_off + kColS + 128u * b;
         float s[128];
@@ -406,8 +403,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         if (j == 0) {
           m_run = m_tile;
         } else if (__any_sync(0xffffffffu, m_tile > m_run + 8.0f)) {
-          // O must first hold P_t-1 V_t-1: pair t - 1 complete
-          if (!wait_pair(t - 1, 9)) goto softmax_done;
+          // O must first hold P_j-1 V_j-1: group G + j + 1 complete
+          if (!wait_group(G + j + 1, 9)) goto softmax_done;
           tc_fence_after();
           const float m_new = fmaxf(m_run, m_tile);
           const float alpha = ex2_approx(m_run - m_new);
@@ -458,10 +455,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
           l_run += lo + hi;
         }
         // the MMA thread waits only for P: the leader's warp 0 first makes
-        // sure that pair t's ring stage (t + 2) has landed
+        // sure that the stage of P_j V_j's group (G + j + 2) has landed
         if (leader && warp == 0 &&
-            !wait_warp(bar(L::kStageFull + ((t + 2) & (kStages - 1))), static_cast<uint32_t>((t + 2) / kStages) & 1u,
-                       ctl, 13))
+            !wait_warp(bar(L::kStageFull + ((G + j + 2) & (kStages - 1))), group_parity(G + j + 2), ctl, 13))
           goto softmax_done;
         tmem_wait_st();
         tc_fence_before();
@@ -469,7 +465,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         if (lane == 0) mbar_arrive_cluster(mapa_shared(bar(L::kPFull + b), 0));
       }
       {
-        if (!wait_pair(t - 1, 10)) goto softmax_done;  // the item's last pair
+        if (!wait_group(G + nkv + 1, 10)) goto softmax_done;  // the item's last group
         tc_fence_after();
         const float inv_l = 1.0f / l_run;
         const uint32_t t_o = tmem + lane_off + kColO;
@@ -495,6 +491,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
           if (args.lse) args.lse[grow * args.num_heads + head] = (m_run + log2f(l_run)) * 0.69314718055994530942f;
         }
       }
+      G += nkv + 2;
     }
   softmax_done:;
   }
