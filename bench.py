@@ -37,6 +37,40 @@ METRIC = "cached-ref attention TFLOP/s & ms/step (5 refs,1024²); modelled 40-st
 UNIT = "TFLOP/s"
 T_STEPS = 40
 N_LIVE_SETS = 4
+# ncu record of DRAM bytes per step-attention launch (1024^2, 5 references),
+# valid only for the kernel sources it was taken with
+TRAFFIC_RECORD = os.path.join(ROOT, "profiles", "attn_tc2_kernel_step_edit1024_5ref_traffic.txt")
+KERNEL_SOURCES = ("attn_tc2.cuh", "attn_tc.cuh", "common.cuh", "ptx.cuh")
+
+
+def kernel_source_hash() -> str:
+    import hashlib
+
+    h = hashlib.sha256()
+    for name in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_2608_21229_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+def recorded_traffic(workload: str, kernel: str):
+    """DRAM bytes per launch from the committed ncu record, or None when the
+    record is missing, is for another workload or kernel, or predates the
+    current kernel sources."""
+    if workload != "edit1024_5ref" or kernel != "tcgen05" or not os.path.exists(TRAFFIC_RECORD):
+        return None
+    fields = {}
+    with open(TRAFFIC_RECORD) as f:
+        for line in f:
+            if ":" in line and not line.startswith((" ", "#", "|")):
+                k, v = line.split(":", 1)
+                fields[k.strip()] = v.strip()
+    if fields.get("kernel_source_sha256") != kernel_source_hash():
+        return None
+    try:
+        return float(fields["dram_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
 
 
 def peaks():
@@ -250,12 +284,16 @@ def run_ours(args, ws, rank, local):
             "paper_end_to_end": {"5_refs": 3.92, "10_refs": 5.47, "note": "whole model, unnamed GPU (context)"},
         },
         "roofline": {
-            "kernel": f"attn_{args.kernel}_kernel<{D}> (step_attention)",
+            "kernel": ("attn_mma_kernel (mma.sync)" if args.kernel == "mma_sync" else
+                       "attn_tc2_kernel (tcgen05, CTA pairs)" if D == 128 else "attn_tc_kernel<64> (tcgen05)")
+                      + " in step_attention",
             "bound": "tensor", "achieved": achieved, "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
             "frac": achieved / pk["bf16_sustained"],
             "peak_kind": f"bf16 dense, {pk['source']} sustained (kernel timed inside a long step)",
             "frac_of_burst": achieved / pk["bf16_burst"],
-            "traffic": None,
+            "traffic": recorded_traffic(w.name, args.kernel),
+            "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum, one step_attention launch"
+                              " (profiles/); null when the kernel sources changed since",
             "algorithmic_bytes": 2 * (seg.live_rows * H * D * 2) * 2 + acc.cache_bytes(w.requests, H, D),
         },
         "e2e": e2e,
