@@ -246,6 +246,9 @@ def run_ours(args, ws, rank, local):
     if not args.no_full:
         t_full = time_full(w, dev, stream, scale)
     e2e = None if args.no_e2e else run_e2e(args, w, cache, seg, dev, stream, scale, flops_per_step)
+    cfg = None
+    if w.name == "edit1024_5ref" and not args.no_cfg:
+        cfg = time_cfg_pair(dev, stream, scale, t_step)
     flops_all, secs_all = aggregate(flops_per_step * args.steps, total_s, ws)
     pk = peaks()
     achieved = step_flops / t_step / 1e12
@@ -296,6 +299,7 @@ def run_ours(args, ws, rank, local):
                               " (profiles/); null when the kernel sources changed since",
             "algorithmic_bytes": 2 * (seg.live_rows * H * D * 2) * 2 + acc.cache_bytes(w.requests, H, D),
         },
+        "cfg_pair": cfg,
         "e2e": e2e,
         "clocks": clk.summary(),
         "gpu_launches": launches_per_step * args.steps,
@@ -303,6 +307,50 @@ def run_ours(args, ws, rank, local):
     if rank == 0 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget)
     return line
+
+
+def time_cfg_pair(dev, stream, scale, t_step_positive):
+    """Step attention of a guided generation: the positive and the negative
+    (blank-text) branch of the headline edit as two requests of one launch."""
+    import torch
+
+    import workloads
+    from paper_2608_21229_gb300 import accounting as acc
+    from paper_2608_21229_gb300 import refcache as rcb
+
+    w = workloads.CFG_1024_5REF
+    H, D = w.num_heads, w.head_dim
+    seg = rcb.Segments.from_workload(w)
+    cache = rcb.RefCache(seg, num_layers=1, mask_mode="beyond", device=dev)
+    qs, ks, vs = (t.to(dev) for t in workloads.static_qkv(w))
+    lives = [tuple(t.to(dev) for t in workloads.live_qkv(w, step=i)) for i in range(N_LIVE_SETS)]
+    o_s = torch.empty(seg.static_rows, H, D, dtype=torch.bfloat16, device=dev)
+    o_l = torch.empty(seg.live_rows, H, D, dtype=torch.bfloat16, device=dev)
+    cache.build(0, qs, ks, vs, o_s, scale=scale)
+    for i in range(3):
+        cache.step(0, *lives[i % N_LIVE_SETS], o_l, scale=scale)
+    n = 2 * T_STEPS
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for i in range(n):
+        cache.step(0, *lives[i % N_LIVE_SETS], o_l, scale=scale)
+    b.record(stream)
+    torch.cuda.synchronize()
+    if rcb.status() != rcb.OK:
+        raise RuntimeError(f"device error in the guided step: {rcb.last_error()}")
+    t = a.elapsed_time(b) / n / 1e3
+    flops = acc.flops(acc.step_units(w.requests), H, D)
+    return {
+        "workload": w.name,
+        "requests": [[x.n_st, x.n_lt, x.n_x, x.n_r] for x in w.requests],
+        "step_ms": t * 1e3,
+        "tflops": flops / t / 1e12,
+        "flops": flops,
+        "vs_positive_branch_alone": t / t_step_positive,
+        "interaction_model_40step": acc.modelled_ratio(w.requests, T_STEPS),
+        "note": "both branches of true CFG (App. D) in one step_attention launch; "
+                "the negative branch has no instruction tokens and its own cache",
+    }
 
 
 def time_full(w, dev, stream, scale):
@@ -482,6 +530,7 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end measurement")
     ap.add_argument("--no-full", action="store_true", help="skip the full-attention baseline")
+    ap.add_argument("--no-cfg", action="store_true", help="skip the guided (positive + negative branch) step")
     args = ap.parse_args(argv)
     ws, rank, local = dist_env()
     if args.warmup < 3:

@@ -204,3 +204,33 @@ def test_not_built_and_bad_args_are_rejected():
         cache.build(0, mis, ks, vs, os_)
     assert e.value.code == rcb.ERR_INVALID_ARG
     assert rcb.status() == rcb.OK
+
+
+# ---------------------------------------------------------------- CFG pair (positive + negative branch)
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_cfg_small_full_compare(kernel):
+    run = pu.GpuRun(workloads.CFG_SMALL, kernel=kernel)
+    pu.full_compare(run)
+
+
+def test_cfg_edit1024_5ref_sampled():
+    run = pu.GpuRun(workloads.CFG_1024_5REF, kernel="tcgen05")
+    pu.sampled_compare(run, seed=9, per_request=24)
+
+
+@pytest.mark.parametrize("w", [workloads.CFG_SMALL, workloads.CFG_1024_5REF], ids=lambda w: w.name)
+def test_cfg_pair_equals_branches_run_alone_bitwise(w):
+    """Both branches in one launch give, bit for bit, what each branch gives alone."""
+    pair = pu.GpuRun(w, kernel="tcgen05")
+    for b, r in enumerate(w.requests):
+        single = workloads.Workload(f"{w.name}_branch{b}", w.num_heads, w.head_dim, (r,), w.seed)
+        s0, l0 = w.cu_static[b], w.cu_live[b]
+        static = tuple(t[s0:s0 + r.n_static] for t in pair.static)
+        live = tuple(t[l0:l0 + r.n_live] for t in pair.live)
+        alone = pu.GpuRun(single, kernel="tcgen05", static=static, live=live)
+        assert np.array_equal(pu.bits(alone.o_live), pu.bits(pair.o_live[l0:l0 + r.n_live]))
+        assert np.array_equal(pu.bits(alone.o_static), pu.bits(pair.o_static[s0:s0 + r.n_static]))
+        assert np.array_equal(alone.lse_live.cpu().numpy(), pair.lse_live[l0:l0 + r.n_live].cpu().numpy())
+        c0 = pu.cache_offsets(w, "beyond")[b]
+        assert np.array_equal(pu.bits(alone.k_cache), pu.bits(pair.k_cache[c0:c0 + r.n_r]))
+        assert np.array_equal(pu.bits(alone.v_cache), pu.bits(pair.v_cache[c0:c0 + r.n_r]))

@@ -108,7 +108,17 @@ RAGGED_4REQ = _w(
     3,
 )
 
-ALL = {w.name: w for w in (TINY, EDIT_512_2REF, EDIT_1024_5REF, RAGGED_4REQ) + SWEEP_1024}
+#: True classifier-free guidance (App. D, Sampling: gamma = 4 with a blank
+#: negative prompt) runs a positive and a negative branch every step.  The
+#: negative branch keeps the references and the target and has only the text
+#: emptied (App. E): no live instruction tokens, and an anchor block of blank
+#: text, so its reference cache differs from the positive branch's and is a
+#: request of its own.  Both branches run as two requests of one ragged batch,
+#: one launch per call.
+CFG_1024_5REF = _w("cfg_edit1024_5ref", 24, 128, [(128, 512, 4096, 5 * 4096), (128, 0, 4096, 5 * 4096)], 4)
+CFG_SMALL = _w("cfg_small", 4, 128, [(32, 64, 512, 1024), (32, 0, 512, 1024)], 5)
+
+ALL = {w.name: w for w in (TINY, EDIT_512_2REF, EDIT_1024_5REF, RAGGED_4REQ, CFG_1024_5REF, CFG_SMALL) + SWEEP_1024}
 
 
 def _fnv1a(text: str) -> int:
