@@ -13,13 +13,16 @@
 // CTA keeps its own 128 query rows (A is split along M).  Per SM this halves
 // the tile bytes fetched and the B-operand bytes read, for the same MMA work.
 //
-// Cluster of 2 CTAs (rank 0 = leader), 192 threads each:
+// Cluster of 2 CTAs (rank 0 = leader), 224 threads each:
 //   warps 0-3  softmax: thread l of warp w owns row 32 w + l of this CTA's
 //              128 rows (its TMEM lane), all 128 score columns of a tile
 //   warp 4     TMA producer: this CTA's Q rows and its halves of the K and V
 //              tiles; completion is counted on the leader's barriers
 //   warp 5     both CTAs: TMEM allocation (a pair operation); leader only:
-//              the MMA thread
+//              the MMA warp (lane 0 issues every MMA and commit)
+//   warp 6     leader only: the gate warp, which does every mbarrier wait
+//              the MMAs depend on and hands each group to the MMA warp
+//              through a named barrier
 // One softmax warp per SM sub-partition leaves the MMA warp's sub-partition
 // with a single busy warp beside it, and a row needs no partner thread.
 // An item is a task of up to 256 query rows: CTA r takes rows
@@ -38,8 +41,13 @@
 // Synchronisation is built so that the MMA thread does as little as possible
 // between its MMAs: a tcgen05.mma blocks its thread until the tensor core
 // takes it, and the tensor core queues almost nothing, so every cycle the
-// MMA thread spends between two groups idles the tensor core.  Per group the
-// MMA thread waits once (P ready) and commits once:
+// MMA thread spends between two groups idles the tensor core.  An mbarrier
+// wait whose result the MMA thread needs costs it far more than a
+// named-barrier handshake, so all mbarrier waits are done by the gate warp:
+// per group, the gate warp waits for what the group needs and then meets the
+// MMA warp at `bar.red.or` (which also carries an abort bit: both warps walk
+// the same group sequence and leave together, so neither can be left waiting);
+// the MMA thread then issues the group and commits once:
 //   pair_done[g % 4]   one commit per group (multicast to both CTAs): its S
 //                      is in TMEM, its P.V is in O, its stage and the P
 //                      buffer it read are free.  Four barriers, so that no
@@ -60,7 +68,7 @@ namespace rc {
 namespace tc2 {
 using tc::Ctl;
 constexpr int kD = 128;
-constexpr int kThreads = 192;
+constexpr int kThreads = 224;
 constexpr int kStages = 4;                  // ring stages (pair_done has as many barriers)
 constexpr uint32_t kKHalf = 64 * 128 * 2;   // 16 KB: this CTA's 64 keys x 128 d of a K tile
 constexpr uint32_t kVHalf = 128 * 64 * 2;   // 16 KB: 128 keys x this CTA's 64 d of a V tile
@@ -68,7 +76,8 @@ constexpr uint32_t kStage = kKHalf + kVHalf;
 constexpr uint32_t kQTile = 128 * 128 * 2;
 constexpr uint32_t kKBox = 64 * 128;        // one K box: 64 rows x 128 bytes
 constexpr int kWarpArrivals = 8;            // 4 softmax warps in each of the 2 CTAs
-constexpr int kProducerWarp = 4, kMmaWarp = 5;
+constexpr int kProducerWarp = 4, kMmaWarp = 5, kGateWarp = 6;
+constexpr uint32_t kGateBarrier = 1;  // named barrier of the MMA and gate warps (0 is __syncthreads)
 static_assert(kStages == 4, "pair_done indexing assumes four stages");
 
 struct Smem {
@@ -252,8 +261,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
     }
     __syncwarp();
   } else if (warp == tc2::kMmaWarp) {
-    // ------------------------------------------------------------ MMA issuer (leader)
-    if (leader && lane == 0) {
+    // ------------------------------------------------------------ MMA warp (leader)
+    if (leader) {
       // descriptors of stage 0 (stage s: + s * kStage / 16) and of Q buffer 0
       const uint64_t kd0 = sdesc_sw128(base + L::kRing, 16, 1024);
       const uint64_t vd0 = sdesc_sw128(base + L::kRing + kKHalf, kBoxBytes, 1024);
@@ -274,60 +283,93 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         const int nkv = n_key_tiles(tk, na);
         if (nkv == 0) continue;
         const int qb = qi & 1;
-        if (!wait_one(bar(L::kQFull + qb), static_cast<uint32_t>(qi >> 1) & 1u, ctl, 3)) goto mma_done;
         const uint64_t qd = qdesc0 + ((static_cast<uint32_t>(qb) * kQTile) >> 4);
-        // groups G, G + 1: S_0, S_1
+        // groups G, G + 1: S_0, S_1 (the gate warp has seen the Q tile and stage g land)
         for (int n = 0; n < 2; ++n, ++g) {
+          if (bar_red_or(tc2::kGateBarrier, 64, false)) goto mma_done;
           const int slot = g & (kStages - 1);
-          if (!wait_one(bar(L::kStageFull + slot), group_parity(g), ctl, 4)) goto mma_done;
-          if (n < nkv) {
-            tc_fence_after();
-            const uint64_t kd = kd0 + static_cast<uint64_t>(slot) * (kStage >> 4);
-            const uint32_t d_s = tmem + kColS + (static_cast<uint32_t>((t0 + n) & 1) << 7);
+          if (lane == 0) {
+            if (n < nkv) {
+              tc_fence_after();
+              const uint64_t kd = kd0 + static_cast<uint64_t>(slot) * (kStage >> 4);
+              const uint32_t d_s = tmem + kColS + (static_cast<uint32_t>((t0 + n) & 1) << 7);
 #pragma unroll
-            for (int kk = 0; kk < D / 16; ++kk) tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
-            issued = true;
-            if (n == nkv - 1) tc2_commit_mc(bar(L::kQEmpty + qb), 3);
-          }
-          tc2_commit_mc(bar(L::kPairDone + slot), 3);
-        }
-        // groups G + 2 + j: P_j V_j (+ S_j+2)
-        for (int j = 0; j < nkv; ++j, ++g) {
-          const int t = t0 + j;
-          // P_t ready: also covers this group's stage and the previous item's O reads
-          if (!wait_cl(bar(L::kPFull + (t & 1)), static_cast<uint32_t>(t >> 1) & 1u, ctl, 7)) goto mma_done;
-          tc_fence_after();
-          const int slot = g & (kStages - 1);
-          const uint64_t soff = static_cast<uint64_t>(slot) * (kStage >> 4);
-          const uint64_t vd = vd0 + soff;
-          const uint32_t a_p = tmem + kColP + (static_cast<uint32_t>(t & 1) << 6);
-          const uint32_t acc0 = j > 0 ? 1u : 0u;
-          if (j + 2 < nkv) {
-            const uint64_t kd = kd0 + soff;
-            const uint32_t d_s = tmem + kColS + (static_cast<uint32_t>(t & 1) << 7);
-#pragma unroll
-            for (int kk = 0; kk < 8; ++kk) {
-              tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, kk > 0 ? 1u : acc0);
-              tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
+              for (int kk = 0; kk < D / 16; ++kk)
+                tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
+              if (n == nkv - 1) tc2_commit_mc(bar(L::kQEmpty + qb), 3);
             }
-            if (j + 2 == nkv - 1) tc2_commit_mc(bar(L::kQEmpty + qb), 3);
-          } else {
-#pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
-              tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, kk > 0 ? 1u : acc0);
+            tc2_commit_mc(bar(L::kPairDone + slot), 3);
           }
-          tc2_commit_mc(bar(L::kPairDone + slot), 3);
+          issued = true;
+          __syncwarp();
+        }
+        // groups G + 2 + j: P_j V_j (+ S_j+2) (the gate warp has seen P_t, which
+        // also covers this group's stage and the previous item's O reads)
+        for (int j = 0; j < nkv; ++j, ++g) {
+          if (bar_red_or(tc2::kGateBarrier, 64, false)) goto mma_done;
+          if (lane == 0) {
+            const int t = t0 + j;
+            tc_fence_after();
+            const int slot = g & (kStages - 1);
+            const uint64_t soff = static_cast<uint64_t>(slot) * (kStage >> 4);
+            const uint64_t vd = vd0 + soff;
+            const uint32_t a_p = tmem + kColP + (static_cast<uint32_t>(t & 1) << 6);
+            const uint32_t acc0 = j > 0 ? 1u : 0u;
+            if (j + 2 < nkv) {
+              const uint64_t kd = kd0 + soff;
+              const uint32_t d_s = tmem + kColS + (static_cast<uint32_t>(t & 1) << 7);
+#pragma unroll
+              for (int kk = 0; kk < 8; ++kk) {
+                tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, kk > 0 ? 1u : acc0);
+                tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
+              }
+              if (j + 2 == nkv - 1) tc2_commit_mc(bar(L::kQEmpty + qb), 3);
+            } else {
+#pragma unroll
+              for (int kk = 0; kk < 8; ++kk)
+                tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, kk > 0 ? 1u : acc0);
+            }
+            tc2_commit_mc(bar(L::kPairDone + slot), 3);
+          }
+          __syncwarp();
         }
         t0 += nkv;
         ++qi;
       }
     mma_done:
-      if (issued) {  // every MMA must finish before TMEM is freed
+      if (issued && lane == 0) {  // every MMA must finish before TMEM is freed
         tc2_commit_mc(bar(L::kMmaDone), 1);
         drain_one(bar(L::kMmaDone), 0u, args.timeout_ns);
       }
     }
     __syncwarp();
+  } else if (warp == tc2::kGateWarp) {
+    // ------------------------------------------------------------ gate warp (leader)
+    // The same group sequence as the MMA warp; every wait is bounded, and a
+    // failed wait is passed on through the handshake, after which both leave.
+    if (leader) {
+      int g = 0, t0 = 0, qi = 0;
+      for (int item = cluster; item < args.n_items; item += n_clusters) {
+        Task tk;
+        int head, na;
+        decode_item(args, item, tk, head);
+        const int nkv = n_key_tiles(tk, na);
+        if (nkv == 0) continue;
+        bool ok = wait_cl_warp(bar(L::kQFull + (qi & 1)), static_cast<uint32_t>(qi >> 1) & 1u, ctl, 3);
+        for (int n = 0; n < 2; ++n, ++g) {
+          ok = ok && wait_cl_warp(bar(L::kStageFull + (g & (kStages - 1))), group_parity(g), ctl, 4);
+          if (bar_red_or(tc2::kGateBarrier, 64, !ok)) goto gate_done;
+        }
+        for (int j = 0; j < nkv; ++j, ++g) {
+          const int t = t0 + j;
+          ok = wait_cl_warp(bar(L::kPFull + (t & 1)), static_cast<uint32_t>(t >> 1) & 1u, ctl, 7);
+          if (bar_red_or(tc2::kGateBarrier, 64, !ok)) goto gate_done;
+        }
+        t0 += nkv;
+        ++qi;
+      }
+    gate_done:;
+    }
   } else {
     // ------------------------------------------------------------ softmax (both CTAs)
     const int trow = warp * 32 + lane;                     // row within this CTA's 128 rows (= TMEM lane)

@@ -259,6 +259,22 @@ __device__ __forceinline__ void tc2_commit_mc(uint32_t bar, uint16_t cta_mask) {
       : "memory");
 }
 
+// ---------------------------------------------------------------- named barriers
+// Named barrier `id` over `nthreads` threads (whole warps, all lanes of each
+// participating warp execute it); returns the OR of every thread's `pred`.
+__device__ __forceinline__ bool bar_red_or(uint32_t id, uint32_t nthreads, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred pi, po;\n\t"
+      "setp.ne.u32 pi, %1, 0;\n\t"
+      "bar.red.or.pred po, %2, %3, pi;\n\t"
+      "selp.u32 %0, 1, 0, po;\n\t}"
+      : "=r"(r)
+      : "r"(pred ? 1u : 0u), "r"(id), "r"(nthreads)
+      : "memory");
+  return r != 0;
+}
+
 // ---------------------------------------------------------------- descriptors
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, bool b_mn_major) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
