@@ -170,6 +170,26 @@ def aggregate(local_flops: float, local_seconds: float, world_size: int):
 
 
 # ----------------------------------------------------------------------------- our arm
+def workload_config(w, kernel: str, ws: int) -> dict:
+    """`config` of the bench line (both arms): the workload and how it is run."""
+    from paper_2608_21229_gb300 import accounting as acc
+
+    H, D = w.num_heads, w.head_dim
+    live_rows = w.cu_live[-1]
+    cache_b = acc.cache_bytes(w.requests, H, D)
+    live_b = 3 * live_rows * H * D * 2
+    return {
+        "workload": w.name, "num_heads": H, "head_dim": D,
+        "requests": [[x.n_st, x.n_lt, x.n_x, x.n_r] for x in w.requests],
+        "segments": "(N_ST, N_LT, N_X, N_R) per request",
+        "step": f"refcache_build + {T_STEPS} step_attention (one layer, one generation)",
+        "mask": "beyond (Sec. 3.3)", "kernel": kernel,
+        "l2": ("inputs larger than L2" if cache_b + live_b > 129e6 else "inputs smaller than L2 (not flushed)")
+              + f": {cache_b / 1e6:.0f} MB cache + {N_LIVE_SETS} live Q/K/V sets of {live_b / 1e6:.0f} MB cycled",
+        "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU",
+    }
+
+
 def run_ours(args, ws, rank, local):
     import torch
 
@@ -265,18 +285,7 @@ def run_ours(args, ws, rank, local):
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic",
-        "config": {
-            "workload": w.name, "num_heads": H, "head_dim": D,
-            "requests": [[x.n_st, x.n_lt, x.n_x, x.n_r] for x in w.requests],
-            "segments": "(N_ST, N_LT, N_X, N_R) per request",
-            "step": f"refcache_build + {T_STEPS} step_attention (one layer, one generation)",
-            "mask": "beyond (Sec. 3.3)", "kernel": args.kernel,
-            "l2": ("inputs larger than L2" if acc.cache_bytes(w.requests, H, D) + 3 * seg.live_rows * H * D * 2
-                   > 129e6 else "inputs smaller than L2 (not flushed)")
-                  + f": {acc.cache_bytes(w.requests, H, D) / 1e6:.0f} MB cache + "
-                  f"{N_LIVE_SETS} live Q/K/V sets of {3 * seg.live_rows * H * D * 2 / 1e6:.0f} MB cycled",
-            "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU",
-        },
+        "config": workload_config(w, args.kernel, ws),
         "step_attention": {"ms": t_step * 1e3, "tflops": achieved, "flops": step_flops},
         "prefill": {"ms": t_pre * 1e3, "tflops": pre_flops / t_pre / 1e12, "flops": pre_flops},
         "full_attention": {"ms": t_full * 1e3, "tflops": full_flops / t_full / 1e12, "flops": full_flops}
@@ -543,7 +552,7 @@ def run_reference(args, ws, rank):
     return {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": tot_s / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-            "config": {"workload": w.name, "note": "CPU oracle (plain fp64 definition) on bounded samples"},
+            "config": workload_config(w, "cpu oracle (plain fp64 definition) on bounded samples", ws),
             "cpu_baseline": {"value": v, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
