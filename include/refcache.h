@@ -40,9 +40,13 @@
  *     refcache_status().
  *   - Host arrays (segment tables) are read during the call only; the library
  *     keeps its own copies.
- *   - No entry point allocates device memory except refcache_create (unless it
- *     is given memory) and full_attention (a per-device work-list buffer that
- *     it keeps and grows).
+ *   - No entry point allocates device memory except refcache_create (the
+ *     cache, unless it is given memory, and for head_dim 128 a separate work
+ *     list with a workspace for split items, see refcache_create) and
+ *     full_attention (a per-device work-list buffer that it keeps and grows).
+ *   - The refcache_build and step_attention calls of one cache share that
+ *     workspace: issue them in stream order (one stream, or streams ordered
+ *     by events), not concurrently.
  */
 #ifndef REFCACHE_H
 #define REFCACHE_H
@@ -122,6 +126,14 @@ REFCACHE_API size_t refcache_bytes(int num_layers, int mask_mode, const refcache
  * with cudaMalloc on the current device and frees it in refcache_destroy;
  * otherwise it uses dev_mem (>= refcache_bytes(), 256-byte aligned, owned by
  * the caller, not freed).  Synchronous.  *out is set only on success.
+ *
+ * For head_dim 128 it also plans, for the current device, the per-item work
+ * lists of the prefill and the step: when their (query tile, head) items do
+ * not fill the last round of the GPU's CTA pairs evenly, the items of that
+ * round are split by key range into 2-8 parts whose outputs a combine kernel
+ * merges.  These lists and an fp32 workspace for the parts (parts x 256 rows
+ * x (head_dim + 1) x 4 bytes, e.g. 27 MB at 1024^2 with five references) are
+ * one more cudaMalloc, freed by refcache_destroy.
  */
 REFCACHE_API int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refcache_segments_t* seg,
                     void* dev_mem, size_t dev_bytes);

@@ -1,0 +1,72 @@
+// attn_combine.cuh -- merge the parts of split items.
+//
+// When the items of a launch do not divide evenly over the GPU's CTA pairs,
+// the last items are split by key range into parts that run on otherwise idle
+// pairs.  Each part p of an item leaves, for every query row, its own
+// normalised output O_p = (sum_j p_j v_j) / l_p and L_p = m_p + log l_p over
+// its keys.  Over all keys of the item the softmax normaliser is
+// l = sum_p exp(L_p), so the item's output is
+//   O = sum_p exp(L_p - L) O_p   with   L = log sum_p exp(L_p),
+// computed here with L_max subtracted first: one warp per query row, four
+// head-dim columns per lane.
+#pragma once
+#include <cuda_bf16.h>
+
+#include "common.cuh"
+
+namespace rc {
+
+constexpr int kMaxParts = 8;
+
+// grid = (ceil(rows / 8), jobs), 256 threads: one warp per query row, all
+// parts' loads issued before any is used.
+template <int D>
+__global__ void __launch_bounds__(256) combine_parts_kernel(const CombineJob* __restrict__ jobs,
+                                                            const float* __restrict__ part_o,
+                                                            const float* __restrict__ part_lse, int rows_per_part,
+                                                            __nv_bfloat16* __restrict__ out, float* __restrict__ lse,
+                                                            int64_t row_stride, int num_heads) {
+  static_assert(D == 128, "four columns per lane");
+  const CombineJob job = jobs[blockIdx.y];
+  const int r = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (r >= job.q_rows) return;
+  const int np = min(job.nparts, kMaxParts);
+  float L[kMaxParts];
+  float4 v[kMaxParts];
+#pragma unroll
+  for (int p = 0; p < kMaxParts; ++p) {
+    if (p < np) {
+      const int64_t row = static_cast<int64_t>(job.part0 + p) * rows_per_part + r;
+      L[p] = part_lse[row];
+      v[p] = reinterpret_cast<const float4*>(part_o + row * D)[lane];
+    } else {
+      L[p] = -INFINITY;
+      v[p] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  }
+  float lmax = L[0];
+#pragma unroll
+  for (int p = 1; p < kMaxParts; ++p) lmax = fmaxf(lmax, L[p]);
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  float wsum = 0.f;
+#pragma unroll
+  for (int p = 0; p < kMaxParts; ++p) {
+    const float w = p < np ? expf(L[p] - lmax) : 0.f;
+    wsum += w;
+    acc[0] += w * v[p].x;
+    acc[1] += w * v[p].y;
+    acc[2] += w * v[p].z;
+    acc[3] += w * v[p].w;
+  }
+  const float inv = 1.0f / wsum;
+  const int64_t row = static_cast<int64_t>(job.q_row0) + r;
+  __nv_bfloat162 lo = __floats2bfloat162_rn(acc[0] * inv, acc[1] * inv);
+  __nv_bfloat162 hi = __floats2bfloat162_rn(acc[2] * inv, acc[3] * inv);
+  uint2 packed;
+  packed.x = *reinterpret_cast<uint32_t*>(&lo);
+  packed.y = *reinterpret_cast<uint32_t*>(&hi);
+  reinterpret_cast<uint2*>(out + row * row_stride + static_cast<int64_t>(job.head) * D)[lane] = packed;
+  if (lse && lane == 0) lse[row * num_heads + job.head] = lmax + logf(wsum);
+}
+
+}  // namespace rc

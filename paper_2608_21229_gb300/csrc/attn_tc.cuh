@@ -137,8 +137,14 @@ __device__ __forceinline__ TileSrc tile_src(const Task& t, int na, int j) {
 
 // Items are enumerated head-major (item = head * n_tasks + task, tasks
 // longest first): CTAs that run at the same time then work on few heads, so
-// the K/V tiles they all stream stay in L2.
+// the K/V tiles they all stream stay in L2.  A per-item list is already in
+// that order and names the head of every item.
 __device__ __forceinline__ void decode_item(const AttnArgs& a, int item, Task& t, int& head) {
+  if (a.per_item) {
+    t = a.tasks[item];
+    head = t.head;
+    return;
+  }
   head = item / a.n_tasks;
   t = a.tasks[item - head * a.n_tasks];
 }

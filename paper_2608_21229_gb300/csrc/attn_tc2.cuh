@@ -511,6 +511,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         tc_fence_after();
         const float inv_l = 1.0f / l_run;
         const uint32_t t_o = tmem + lane_off + kColO;
+        if (tk.part > 0) {
+          // a part of a split item: O / l in fp32 and m + log l to its workspace slot
+          const int64_t prow_ws = static_cast<int64_t>(tk.part - 1) * args.rows_per_task + prow;
+          float4* dst = reinterpret_cast<float4*>(args.part_o + prow_ws * D);
+#pragma unroll
+          for (int cc = 0; cc < D / 32; ++cc) {
+            uint32_t o[32];
+            tmem_ld32(t_o + 32u * cc, o);
+            tmem_wait_ld(o);
+            if (row_ok) {
+#pragma unroll
+              for (int c = 0; c < 8; ++c)
+                dst[8 * cc + c] = make_float4(__uint_as_float(o[4 * c]) * inv_l, __uint_as_float(o[4 * c + 1]) * inv_l,
+                                              __uint_as_float(o[4 * c + 2]) * inv_l,
+                                              __uint_as_float(o[4 * c + 3]) * inv_l);
+            }
+          }
+          tc_fence_before();
+          if (row_ok) args.part_lse[prow_ws] = (m_run + log2f(l_run)) * 0.69314718055994530942f;
+          G += nkv + 2;
+          continue;
+        }
         uint32_t packed[D / 2];
 #pragma unroll
         for (int cc = 0; cc < D / 32; ++cc) {

@@ -10,7 +10,11 @@
 //   full (rows [LT; X_t; R])       A = the request's whole sequence
 // so the mask is never materialised: a key is visible exactly when it lies in
 // A or B, and keys past the end of a range are cut off inside the last tile.
-// A launch enumerates items = tasks x heads, item i -> task i / H, head i % H.
+// A launch enumerates items = tasks x heads, item i -> head i / n_tasks, task
+// i % n_tasks; or, when AttnArgs::per_item is set, an explicit list with one
+// task per item that names its head.  Such a list can also hold *parts* of an
+// item (a sub-range of its key tiles): a part writes its normalised output and
+// log-sum-exp to a workspace slot, and a combine kernel merges the parts.
 #pragma once
 #include <cstdint>
 #include <cuda_bf16.h>
@@ -24,7 +28,8 @@ struct Task {
   int32_t a_len;   //              length
   int32_t b_row0;  // key range B (in the B tensors)
   int32_t b_len;   //              length, 0 = none
-  int32_t pad0, pad1;
+  int32_t head;    // per-item lists only: the item's head
+  int32_t part;    // per-item lists only: 0 = write O, p > 0 = partial result to workspace slot p - 1
 };
 static_assert(sizeof(Task) == 32, "Task layout is part of the device work list");
 
@@ -39,6 +44,9 @@ struct AttnArgs {
   int64_t row_stride;           // elements between rows of Q/K/V/O (= H * D)
   float scale_log2;             // softmax_scale * log2(e)
   int32_t rows_per_task;        // 128 or 256 (the mma.sync kernel splits tasks into 64-row CTAs)
+  int32_t per_item;             // tasks is a per-item list (Task::head, Task::part used)
+  float* part_o;                // workspace of partial results: [slot][rows_per_task][D] fp32, O / l
+  float* part_lse;              //                               [slot][rows_per_task] fp32, m + log l
   uint64_t timeout_ns;          // bound of every in-kernel wait
   // raw pointers, used by the mma.sync kernel (the tcgen05 kernel reads
   // through tensor maps)
@@ -48,6 +56,14 @@ struct AttnArgs {
   const __nv_bfloat16* kb;
   const __nv_bfloat16* vb;
 };
+
+// One item whose key range was split into parts: the combine kernel merges
+// parts [part0, part0 + nparts) of the workspace into rows [q_row0, q_row0 +
+// q_rows) of `head`.
+struct CombineJob {
+  int32_t q_row0, q_rows, head, part0, nparts, pad0, pad1, pad2;
+};
+static_assert(sizeof(CombineJob) == 32, "CombineJob layout is part of the device work list");
 
 // Device error word (one per device that loads the library); kernels set it
 // when a bounded wait runs out, refcache_status() reads and clears it.

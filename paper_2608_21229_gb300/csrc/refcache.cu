@@ -19,8 +19,10 @@
 #include "attn_mma.cuh"
 #include "attn_tc.cuh"
 #include "attn_tc2.cuh"
+#include "attn_combine.cuh"
 
 using rc::AttnArgs;
+using rc::CombineJob;
 using rc::CopySeg;
 using rc::Task;
 
@@ -190,8 +192,9 @@ int launch_tc(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info,
   return REFCACHE_OK;
 }
 
-// The CTA-pair kernel (head_dim 128): grid = 2 x the clusters that fit at once.
-int launch_tc2(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info, cudaStream_t s) {
+// CTA pairs of the head-dim-128 kernel that run at once on this device (the
+// persistent grid); sets the kernel's shared-memory attribute on first use.
+int tc2_clusters(DeviceInfo* info, int* clusters_out) {
   constexpr uint32_t smem = rc::tc2::Smem::kDynamic;
   if (!info->attr_set[4]) {
     cudaError_t e = cudaFuncSetAttribute(rc::attn_tc2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
@@ -206,7 +209,17 @@ int launch_tc2(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info
     info->max_clusters = clusters;
     info->attr_set[4] = true;
   }
-  const int clusters = std::min(a.n_items, info->max_clusters);
+  *clusters_out = info->max_clusters;
+  return REFCACHE_OK;
+}
+
+// The CTA-pair kernel (head_dim 128): grid = 2 x the clusters that fit at once.
+int launch_tc2(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info, cudaStream_t s) {
+  constexpr uint32_t smem = rc::tc2::Smem::kDynamic;
+  int max_clusters = 0;
+  int rc = tc2_clusters(info, &max_clusters);
+  if (rc) return rc;
+  const int clusters = std::min(a.n_items, max_clusters);
   rc::attn_tc2_kernel<<<2 * clusters, rc::tc2::kThreads, smem, s>>>(maps[0], maps[1], maps[2], maps[3], maps[4], a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "attn_tc2_kernel launch");
@@ -239,8 +252,19 @@ struct Operands {
   float* lse;
 };
 
+// A per-item work list with split items (head-dim-128 tcgen05 kernel only):
+// the items, the combine jobs of the split ones and their workspace.
+struct ItemList {
+  const Task* items = nullptr;
+  int n_items = 0;
+  const CombineJob* jobs = nullptr;
+  int n_jobs = 0;
+  float* part_o = nullptr;
+  float* part_lse = nullptr;
+};
+
 int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands& op, float scale, DeviceInfo* info,
-                  cudaStream_t s) {
+                  cudaStream_t s, const ItemList* il = nullptr) {
   if (n_tasks == 0) return REFCACHE_OK;
   AttnArgs a{};
   a.tasks = d_tasks;
@@ -276,7 +300,85 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
     maps[4] = maps[2];
   }
   a.dbg_skip_first_load = g_dbg_skip.exchange(0);
-  return D == 64 ? launch_tc<64>(maps, a, info, s) : launch_tc2(maps, a, info, s);
+  if (D == 64) return launch_tc<64>(maps, a, info, s);
+  if (il && il->items) {
+    a.tasks = il->items;
+    a.per_item = 1;
+    a.n_items = il->n_items;
+    a.part_o = il->part_o;
+    a.part_lse = il->part_lse;
+  }
+  if ((rc = launch_tc2(maps, a, info, s)) != 0) return rc;
+  if (il && il->n_jobs > 0) {
+    const dim3 grid(static_cast<unsigned>((a.rows_per_task + 7) / 8), static_cast<unsigned>(il->n_jobs));
+    rc::combine_parts_kernel<128><<<grid, 256, 0, s>>>(il->jobs, il->part_o, il->part_lse, a.rows_per_task, a.out,
+                                                       a.lse, a.row_stride, H);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "combine_parts_kernel launch");
+  }
+  return REFCACHE_OK;
+}
+
+// Per-item list of `tasks` x heads (head-major, as the kernels enumerate
+// items) for `clusters` CTA pairs.  When the items do not fill the last round
+// of the persistent grid, the items of that round are split by key tiles into
+// s parts each (s chosen so that the parts fill the clusters best), which run
+// after the whole items; their results are merged by combine jobs.
+void plan_items(const std::vector<Task>& tasks, int H, int clusters, std::vector<Task>* items,
+                std::vector<CombineJob>* jobs, int* n_parts) {
+  items->clear();
+  jobs->clear();
+  *n_parts = 0;
+  const int64_t n = static_cast<int64_t>(tasks.size()) * H;
+  if (n == 0 || clusters < 1) return;
+  const int64_t rem = n % clusters;
+  int best_s = 1;
+  double best = 1.0;  // item-times the last round costs
+  if (rem > 0) {
+    for (int cand : {2, 3, 4, 6, 8}) {
+      const double cost = static_cast<double>((rem * cand + clusters - 1) / clusters) / cand;
+      if (cost < best - 1e-9) {
+        best = cost;
+        best_s = cand;
+      }
+    }
+  }
+  const int64_t n_whole = rem > 0 && best_s > 1 ? n - rem : n;
+  std::vector<Task> parts;
+  for (int64_t i = 0; i < n; ++i) {
+    const int h = static_cast<int>(i / static_cast<int64_t>(tasks.size()));
+    Task t = tasks[static_cast<size_t>(i % static_cast<int64_t>(tasks.size()))];
+    t.head = h;
+    t.part = 0;
+    const int na = (t.a_len + 127) / 128, nb = (t.b_len + 127) / 128, nkv = na + nb;
+    const int s_here = std::min(best_s, nkv / 4);  // parts of at least four key tiles
+    if (i < n_whole || s_here < 2) {
+      items->push_back(t);
+      continue;
+    }
+    CombineJob job{};
+    job.q_row0 = t.q_row0;
+    job.q_rows = t.q_rows;
+    job.head = h;
+    job.part0 = *n_parts;
+    job.nparts = s_here;
+    for (int k = 0; k < s_here; ++k) {
+      const int j0 = static_cast<int>(static_cast<int64_t>(nkv) * k / s_here);
+      const int j1 = static_cast<int>(static_cast<int64_t>(nkv) * (k + 1) / s_here);
+      Task p = t;
+      // tiles [j0, j1) of the item's key list (range A, then range B)
+      const int a0 = std::min(j0, na), a1 = std::min(j1, na);
+      p.a_row0 = t.a_row0 + 128 * a0;
+      p.a_len = a1 > a0 ? std::min(t.a_len - 128 * a0, 128 * (a1 - a0)) : 0;
+      const int b0 = std::max(j0, na) - na, b1 = std::max(j1, na) - na;
+      p.b_row0 = t.b_row0 + 128 * b0;
+      p.b_len = b1 > b0 ? std::min(t.b_len - 128 * b0, 128 * (b1 - b0)) : 0;
+      p.part = ++*n_parts;
+      parts.push_back(p);
+    }
+    jobs->push_back(job);
+  }
+  items->insert(items->end(), parts.begin(), parts.end());
 }
 
 // Work list of full_attention_noalloc: a fixed array in static device memory
@@ -310,6 +412,10 @@ struct refcache {
   int n_step = 0;
   CopySeg* d_copy = nullptr;
   int n_copy = 0;
+  // per-item lists of the head-dim-128 kernel with split items, in a separate
+  // allocation: [build items | step items | build jobs | step jobs | part_o | part_lse]
+  uint8_t* aux = nullptr;
+  ItemList build_items, step_items;
   __nv_bfloat16* slots = nullptr;
   int64_t slot_elems = 0;
   std::vector<char> built;
@@ -418,6 +524,58 @@ int check_ptrs(std::initializer_list<const void*> ps, int64_t rows, const char* 
   return REFCACHE_OK;
 }
 
+// Per-item lists (with the last round of items split) for the prefill and
+// the step of a head-dim-128 handle, in one allocation of their own (the
+// caller-sized cache memory is not touched).
+int plan_split_items(refcache* h, DeviceInfo* info, const std::vector<Task>& bt, const std::vector<Task>& st) {
+  int clusters = 0;
+  int rc = tc2_clusters(info, &clusters);
+  if (rc) return rc;
+  std::vector<Task> bi, si;
+  std::vector<CombineJob> bj, sj;
+  int bparts = 0, sparts = 0;
+  plan_items(bt, h->H, clusters, &bi, &bj, &bparts);
+  plan_items(st, h->H, clusters, &si, &sj, &sparts);
+  const int parts = std::max(bparts, sparts);  // build and step calls are stream-ordered: one workspace
+  const int rows = task_rows(h->D);
+  size_t off = 0;
+  const size_t o_bi = off;
+  off = align_up(off + bi.size() * sizeof(Task), 256);
+  const size_t o_si = off;
+  off = align_up(off + si.size() * sizeof(Task), 256);
+  const size_t o_bj = off;
+  off = align_up(off + bj.size() * sizeof(CombineJob), 256);
+  const size_t o_sj = off;
+  off = align_up(off + sj.size() * sizeof(CombineJob), 256);
+  const size_t o_po = off;
+  off = align_up(off + static_cast<size_t>(parts) * rows * h->D * sizeof(float), 256);
+  const size_t o_pl = off;
+  off = align_up(off + static_cast<size_t>(parts) * rows * sizeof(float), 256);
+  cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&h->aux), off);
+  if (e != cudaSuccess) {
+    h->aux = nullptr;
+    return fail(REFCACHE_ERR_OOM, "cudaMalloc(%zu) for the split work lists: %s", off, cudaGetErrorString(e));
+  }
+  auto put = [&](size_t o, const void* src, size_t n) -> cudaError_t {
+    return n ? cudaMemcpy(h->aux + o, src, n, cudaMemcpyHostToDevice) : cudaSuccess;
+  };
+  if ((e = put(o_bi, bi.data(), bi.size() * sizeof(Task))) != cudaSuccess ||
+      (e = put(o_si, si.data(), si.size() * sizeof(Task))) != cudaSuccess ||
+      (e = put(o_bj, bj.data(), bj.size() * sizeof(CombineJob))) != cudaSuccess ||
+      (e = put(o_sj, sj.data(), sj.size() * sizeof(CombineJob))) != cudaSuccess) {
+    cudaFree(h->aux);
+    h->aux = nullptr;
+    return cuda_fail(e, "cudaMemcpy(split work lists)");
+  }
+  float* po = reinterpret_cast<float*>(h->aux + o_po);
+  float* pl = reinterpret_cast<float*>(h->aux + o_pl);
+  h->build_items = ItemList{reinterpret_cast<Task*>(h->aux + o_bi), static_cast<int>(bi.size()),
+                            reinterpret_cast<CombineJob*>(h->aux + o_bj), static_cast<int>(bj.size()), po, pl};
+  h->step_items = ItemList{reinterpret_cast<Task*>(h->aux + o_si), static_cast<int>(si.size()),
+                           reinterpret_cast<CombineJob*>(h->aux + o_sj), static_cast<int>(sj.size()), po, pl};
+  return REFCACHE_OK;
+}
+
 int enter_device(refcache* h, DeviceInfo** info) {
   int dev = 0;
   int rc = current_device(&dev, info);
@@ -491,6 +649,11 @@ int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refca
     delete h;
     return cuda_fail(e, "cudaMemcpy(work tables)");
   }
+  if (h->D == 128 && (rc = plan_split_items(h, info, bt, st)) != 0) {
+    if (h->owns) cudaFree(h->mem);
+    delete h;
+    return rc;
+  }
   h->built.assign(num_layers, 0);
   *out = h;
   return REFCACHE_OK;
@@ -498,12 +661,13 @@ int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refca
 
 void refcache_destroy(refcache_t* h) {
   if (!h) return;
-  if (h->owns && h->mem) {
+  if ((h->owns && h->mem) || h->aux) {
     int prev = 0;
     cudaGetDevice(&prev);
     cudaSetDevice(h->device);
     cudaDeviceSynchronize();
-    cudaFree(h->mem);
+    if (h->owns && h->mem) cudaFree(h->mem);
+    if (h->aux) cudaFree(h->aux);
     cudaSetDevice(prev);
   }
   delete h;
@@ -547,7 +711,8 @@ int refcache_build(refcache_t* h, int layer, const void* q_static, const void* k
     if (e != cudaSuccess) return cuda_fail(e, "copy_rows_kernel launch");
   }
   Operands op{q_static, h->static_rows, k_static, v_static, h->static_rows, nullptr, nullptr, 0, o_static, lse_static};
-  rc = run_attention(h->d_build, h->n_build, h->H, h->D, op, softmax_scale, info, s);
+  rc = run_attention(h->d_build, h->n_build, h->H, h->D, op, softmax_scale, info, s,
+                     h->build_items.items ? &h->build_items : nullptr);
   if (rc) return rc;
   h->built[layer] = 1;
   return REFCACHE_OK;
@@ -565,7 +730,8 @@ int step_attention(refcache_t* h, int layer, const void* q_live, const void* k_l
   void *kslot = nullptr, *vslot = nullptr;
   refcache_kv_ptr(h, layer, &kslot, &vslot, nullptr);
   Operands op{q_live, h->live_rows, k_live, v_live, h->live_rows, kslot, vslot, h->cache_rows, o_live, lse_live};
-  return run_attention(h->d_step, h->n_step, h->H, h->D, op, softmax_scale, info, static_cast<cudaStream_t>(stream));
+  return run_attention(h->d_step, h->n_step, h->H, h->D, op, softmax_scale, info, static_cast<cudaStream_t>(stream),
+                       h->step_items.items ? &h->step_items : nullptr);
 }
 
 int full_attention(int batch, int num_heads, int head_dim, const int32_t* cu_seqlens, const void* q, const void* k,

@@ -118,8 +118,9 @@ def sample_rows(n, rng, extra=24):
     return np.array(sorted(rows), np.int64)
 
 
-def sampled_compare(run: GpuRun, seed=0, per_request=24, scale=None):
-    """Sampled (row, head) outputs of both calls against the oracle, computed one by one."""
+def sampled_compare(run: GpuRun, seed=0, per_request=24, scale=None, heads=None):
+    """Sampled (row, head) outputs of both calls against the oracle, computed
+    one by one; heads restricts the sampled heads."""
     w, mode = run.w, run.mode
     scale = scale or 1.0 / math.sqrt(w.head_dim)
     rng = np.random.default_rng(seed)
@@ -128,14 +129,16 @@ def sampled_compare(run: GpuRun, seed=0, per_request=24, scale=None):
     for b, r in enumerate(w.requests):
         s0, l0 = w.cu_static[b], w.cu_live[b]
         rows = sample_rows(r.n_static, rng, per_request)
-        pairs = np.stack([rows, rng.integers(0, w.num_heads, size=rows.size)], 1).astype(np.int32)
+        hs = rng.choice(np.asarray(heads), size=rows.size) if heads is not None else rng.integers(0, w.num_heads, size=rows.size)
+        pairs = np.stack([rows, hs], 1).astype(np.int32)
         ref_o, ref_l, kc, vc = oracle_static_request(w, mode, b, run.static, scale, pairs)
         check_close(o_s[s0 + pairs[:, 0], pairs[:, 1]], ref_o, l_s[s0 + pairs[:, 0], pairs[:, 1]], ref_l,
                     f"prefill req {b} (sampled)")
         np.testing.assert_array_equal(bits(run.k_cache)[coff[b]:coff[b + 1]], kc)
         np.testing.assert_array_equal(bits(run.v_cache)[coff[b]:coff[b + 1]], vc)
         rows = sample_rows(r.n_live, rng, per_request)
-        pairs = np.stack([rows, rng.integers(0, w.num_heads, size=rows.size)], 1).astype(np.int32)
+        hs = rng.choice(np.asarray(heads), size=rows.size) if heads is not None else rng.integers(0, w.num_heads, size=rows.size)
+        pairs = np.stack([rows, hs], 1).astype(np.int32)
         ref_o, ref_l = oracle_live_request(w, mode, b, run.static, run.live, scale, pairs)
         check_close(o_l[l0 + pairs[:, 0], pairs[:, 1]], ref_o, l_l[l0 + pairs[:, 0], pairs[:, 1]], ref_l,
                     f"step req {b} (sampled)")

@@ -219,8 +219,12 @@ def test_cfg_edit1024_5ref_sampled():
 
 
 @pytest.mark.parametrize("w", [workloads.CFG_SMALL, workloads.CFG_1024_5REF], ids=lambda w: w.name)
-def test_cfg_pair_equals_branches_run_alone_bitwise(w):
-    """Both branches in one launch give, bit for bit, what each branch gives alone."""
+def test_cfg_pair_equals_branches_run_alone(w):
+    """Both branches in one launch give what each branch gives alone: the
+    caches bit for bit, most outputs bit for bit, and every output within a
+    tenth of the parity bar (a launch splits the items of its last round by
+    key range, and which items those are depends on the launch's item count;
+    each part rounds P against its own running maximum)."""
     pair = pu.GpuRun(w, kernel="tcgen05")
     for b, r in enumerate(w.requests):
         single = workloads.Workload(f"{w.name}_branch{b}", w.num_heads, w.head_dim, (r,), w.seed)
@@ -228,9 +232,25 @@ def test_cfg_pair_equals_branches_run_alone_bitwise(w):
         static = tuple(t[s0:s0 + r.n_static] for t in pair.static)
         live = tuple(t[l0:l0 + r.n_live] for t in pair.live)
         alone = pu.GpuRun(single, kernel="tcgen05", static=static, live=live)
-        assert np.array_equal(pu.bits(alone.o_live), pu.bits(pair.o_live[l0:l0 + r.n_live]))
-        assert np.array_equal(pu.bits(alone.o_static), pu.bits(pair.o_static[s0:s0 + r.n_static]))
-        assert np.array_equal(alone.lse_live.cpu().numpy(), pair.lse_live[l0:l0 + r.n_live].cpu().numpy())
+        for got, ref in ((pair.o_live[l0:l0 + r.n_live], alone.o_live),
+                         (pair.o_static[s0:s0 + r.n_static], alone.o_static)):
+            g, a = pu.f64(got), pu.f64(ref)
+            assert np.max(np.abs(g - a)) <= pu.MAX_ABS / 10
+            assert np.mean(pu.bits(got) == pu.bits(ref)) > 0.5
         c0 = pu.cache_offsets(w, "beyond")[b]
         assert np.array_equal(pu.bits(alone.k_cache), pu.bits(pair.k_cache[c0:c0 + r.n_r]))
         assert np.array_equal(pu.bits(alone.v_cache), pu.bits(pair.v_cache[c0:c0 + r.n_r]))
+
+
+# ---------------------------------------------------------------- split items (last round of the persistent grid)
+def test_split_tail_items_sampled():
+    """The last round of items of a launch is split by key range into parts
+    merged by a combine kernel; on the headline case those are items of the
+    last heads (head-major order), for both the prefill and the step."""
+    run = pu.GpuRun(workloads.EDIT_1024_5REF, kernel="tcgen05")
+    pu.sampled_compare(run, seed=21, per_request=64, heads=[21, 22, 23])
+
+
+def test_split_tail_items_cfg_pair_sampled():
+    run = pu.GpuRun(workloads.CFG_1024_5REF, kernel="tcgen05")
+    pu.sampled_compare(run, seed=22, per_request=32, heads=[22, 23])
