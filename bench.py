@@ -217,7 +217,7 @@ def run_ours(args, ws, rank, local):
     step_flops = acc.flops(acc.step_units(w.requests), H, D)
     full_flops = acc.flops(acc.full_units(w.requests), H, D)
     flops_per_step = pre_flops + T_STEPS * step_flops
-    launches_per_step = (1 if acc.cache_bytes(w.requests, H, D) else 0) + 1 + T_STEPS
+    launches_per_step = cache.launches("build") + T_STEPS * cache.launches("step")
 
     def one_step(ev=None):
         if ev is not None:

@@ -152,6 +152,15 @@ REFCACHE_API int refcache_kv_ptr(refcache_t* cache, int layer, void** k_slot, vo
 REFCACHE_API int refcache_layer_built(refcache_t* cache, int layer);
 
 /*
+ * Number of kernels one refcache_build (call = 0) or step_attention (call = 1)
+ * on this cache launches with the kernel family currently selected
+ * (refcache_set_kernel): the attention kernel, the cache copy (build, when
+ * there are cached rows) and the combine of split items (when the cache's
+ * work list has any).  < 0 on error.
+ */
+REFCACHE_API int refcache_call_launches(refcache_t* cache, int call);
+
+/*
  * Static prefill of one layer (Sec. 3.3; cost (N_R + N_ST)^2 per head,
  * Eq. cost-pre).  q_static/k_static/v_static: [cu_static[batch], H, d] bf16,
  * each request's [ST; R] rows.  Writes o_static (same shape) for every ST and

@@ -683,6 +683,16 @@ int refcache_kv_ptr(refcache_t* h, int layer, void** k_slot, void** v_slot, int6
   return REFCACHE_OK;
 }
 
+int refcache_call_launches(refcache_t* h, int call) {
+  if (!h) return fail(REFCACHE_ERR_INVALID_ARG, "cache is NULL");
+  if (call != 0 && call != 1) return fail(REFCACHE_ERR_INVALID_ARG, "call must be 0 (build) or 1 (step)");
+  const int n_tasks = call == 0 ? h->n_build : h->n_step;
+  if (n_tasks == 0) return call == 0 && h->n_copy > 0 ? 1 : 0;
+  const ItemList& il = call == 0 ? h->build_items : h->step_items;
+  const bool tc = g_kernel.load() == REFCACHE_KERNEL_TCGEN05;
+  return (call == 0 && h->n_copy > 0 ? 1 : 0) + 1 + (tc && il.items && il.n_jobs > 0 ? 1 : 0);
+}
+
 int refcache_layer_built(refcache_t* h, int layer) {
   int rc = check_handle_layer(h, layer);
   if (rc) return rc;

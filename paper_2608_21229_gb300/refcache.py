@@ -29,7 +29,7 @@ EXPORTED = (
     "refcache_bytes", "refcache_create", "refcache_destroy", "refcache_kv_ptr", "refcache_layer_built",
     "refcache_build", "step_attention", "full_attention", "refcache_status", "refcache_set_wait_timeout_ns",
     "refcache_set_kernel", "refcache_debug_skip_first_load", "refcache_last_error", "refcache_version",
-    "full_attention_noalloc",
+    "full_attention_noalloc", "refcache_call_launches",
 )
 NOALLOC_MAX_TASKS = 16384
 
@@ -74,6 +74,7 @@ def load(path: Optional[str] = None):
     L.refcache_destroy.restype = None
     L.refcache_kv_ptr.argtypes = [vp, i32, ctypes.POINTER(vp), ctypes.POINTER(vp), ctypes.POINTER(i64)]
     L.refcache_layer_built.argtypes = [vp, i32]
+    L.refcache_call_launches.argtypes = [vp, i32]
     L.refcache_build.argtypes = [vp, i32, vp, vp, vp, vp, vp, f32, vp]
     L.step_attention.argtypes = [vp, i32, vp, vp, vp, vp, vp, f32, vp]
     L.full_attention.argtypes = [i32, i32, i32, ctypes.POINTER(ctypes.c_int32), vp, vp, vp, vp, vp, f32, vp]
@@ -245,6 +246,12 @@ class RefCache:
         r = load().refcache_layer_built(self.h, layer)
         _check(0 if r >= 0 else r)
         return bool(r)
+
+    def launches(self, call: str) -> int:
+        """Kernels one build ('build') or step ('step') call launches."""
+        r = load().refcache_call_launches(self.h, {"build": 0, "step": 1}[call])
+        _check(0 if r >= 0 else r)
+        return int(r)
 
     def build(self, layer, q, k, v, o, lse=None, scale=None, stream=None):
         H, D, n = self.seg.num_heads, self.seg.head_dim, self.seg.static_rows

@@ -254,3 +254,20 @@ def test_split_tail_items_sampled():
 def test_split_tail_items_cfg_pair_sampled():
     run = pu.GpuRun(workloads.CFG_1024_5REF, kernel="tcgen05")
     pu.sampled_compare(run, seed=22, per_request=32, heads=[22, 23])
+
+
+def test_call_launch_counts():
+    """Kernels per call: attention (+ cache copy for the build) (+ combine when
+    the device's plan split the last round; the headline step's 432 items do
+    not fill 76 CTA pairs evenly, so it is split on a GB300)."""
+    w = workloads.EDIT_1024_5REF
+    seg = rcb.Segments.from_workload(w)
+    cache = rcb.RefCache(seg, num_layers=1, mask_mode="beyond")
+    rcb.set_kernel("tcgen05")
+    assert cache.launches("step") in (1, 2)
+    assert cache.launches("build") == cache.launches("step") + 1
+    rcb.set_kernel("mma_sync")
+    assert cache.launches("step") == 1 and cache.launches("build") == 2
+    rcb.set_kernel("tcgen05")
+    tiny = rcb.RefCache(rcb.Segments.from_workload(workloads.TINY), num_layers=1, mask_mode="beyond")
+    assert tiny.launches("step") == 1 and tiny.launches("build") == 2
