@@ -269,6 +269,10 @@ def run_ours(args, ws, rank, local):
     cfg = None
     if w.name == "edit1024_5ref" and not args.no_cfg:
         cfg = time_cfg_pair(dev, stream, scale, t_step)
+    sweep = ragged = None
+    if w.name == "edit1024_5ref" and not args.no_sweep:
+        sweep = [time_step_workload(x, dev, stream, scale) for x in workloads.SWEEP_1024]
+        ragged = time_step_workload(workloads.RAGGED_4REQ, dev, stream, scale)
     flops_all, secs_all = aggregate(flops_per_step * args.steps, total_s, ws)
     pk = peaks()
     achieved = step_flops / t_step / 1e12
@@ -309,6 +313,8 @@ def run_ours(args, ws, rank, local):
             "algorithmic_bytes": 2 * (seg.live_rows * H * D * 2) * 2 + acc.cache_bytes(w.requests, H, D),
         },
         "cfg_pair": cfg,
+        "reference_sweep": sweep,
+        "ragged_batch": ragged,
         "e2e": e2e,
         "clocks": clk.summary(),
         "gpu_launches": launches_per_step * args.steps,
@@ -316,6 +322,72 @@ def run_ours(args, ws, rank, local):
     if rank == 0 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget)
     return line
+
+
+def gpu_randn_bf16(shape, seed: int, dev):
+    """N(0, 1) bf16 drawn on the device from a seeded generator (timing-only
+    inputs; the parity tests use the workloads' CPU draws)."""
+    import torch
+
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+    return torch.randn(shape, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+
+
+def time_step_workload(w, dev, stream, scale, with_full=True):
+    """One workload's step call (and, if asked, its full-attention recompute)
+    timed on its own: build once, then 2 x 40 step calls over four live sets."""
+    import torch
+
+    import workloads
+    from paper_2608_21229_gb300 import accounting as acc
+    from paper_2608_21229_gb300 import refcache as rcb
+
+    H, D = w.num_heads, w.head_dim
+    seg = rcb.Segments.from_workload(w)
+    cache = rcb.RefCache(seg, num_layers=1, mask_mode="beyond", device=dev)
+    qs, ks, vs = (gpu_randn_bf16((seg.static_rows, H, D), 1000 * w.seed + i, dev) for i in range(3))
+    lives = [tuple(gpu_randn_bf16((seg.live_rows, H, D), 1000 * w.seed + 10 + 3 * j + i, dev) for i in range(3))
+             for j in range(N_LIVE_SETS)]
+    o_s = torch.empty(seg.static_rows, H, D, dtype=torch.bfloat16, device=dev)
+    o_l = torch.empty(seg.live_rows, H, D, dtype=torch.bfloat16, device=dev)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    cache.build(0, qs, ks, vs, o_s, scale=scale)
+    for _ in range(2):
+        cache.build(0, qs, ks, vs, o_s, scale=scale)
+    a.record(stream)
+    cache.build(0, qs, ks, vs, o_s, scale=scale)
+    b.record(stream)
+    torch.cuda.synchronize()
+    t_pre = a.elapsed_time(b) / 1e3
+    for i in range(3):
+        cache.step(0, *lives[i % N_LIVE_SETS], o_l, scale=scale)
+    n = 2 * T_STEPS
+    a.record(stream)
+    for i in range(n):
+        cache.step(0, *lives[i % N_LIVE_SETS], o_l, scale=scale)
+    b.record(stream)
+    torch.cuda.synchronize()
+    if rcb.status() != rcb.OK:
+        raise RuntimeError(f"device error in {w.name}: {rcb.last_error()}")
+    t_step = a.elapsed_time(b) / n / 1e3
+    step_flops = acc.flops(acc.step_units(w.requests), H, D)
+    pre_flops = acc.flops(acc.prefill_units(w.requests), H, D)
+    out = {
+        "workload": w.name,
+        "requests": [[x.n_st, x.n_lt, x.n_x, x.n_r] for x in w.requests],
+        "step_ms": t_step * 1e3, "step_tflops": step_flops / t_step / 1e12,
+        "prefill_ms": t_pre * 1e3, "prefill_tflops": pre_flops / t_pre / 1e12,
+        "cache_mb_streamed_per_step": acc.cache_bytes(w.requests, H, D) / 1e6,
+        "interaction_model_40step": acc.modelled_ratio(w.requests, T_STEPS),
+    }
+    del cache
+    if with_full:
+        t_full = time_full(w, dev, stream, scale, gpu_inputs=True)
+        out["full_ms"] = t_full * 1e3
+        out["full_tflops"] = acc.flops(acc.full_units(w.requests), H, D) / t_full / 1e12
+        out["measured_40step"] = acc.measured_ratio(t_full, t_pre, t_step, T_STEPS)
+    return out
 
 
 def time_cfg_pair(dev, stream, scale, t_step_positive):
@@ -362,7 +434,7 @@ def time_cfg_pair(dev, stream, scale, t_step_positive):
     }
 
 
-def time_full(w, dev, stream, scale):
+def time_full(w, dev, stream, scale, gpu_inputs=False):
     """Seconds per full_attention call over every request's [LT; X; R]."""
     import torch
 
@@ -374,7 +446,10 @@ def time_full(w, dev, stream, scale):
     for x in w.requests:
         cu_full.append(cu_full[-1] + x.n_lt + x.n_x + x.n_r)
     n_full = cu_full[-1]
-    qf, kf, vf = (workloads.randn_bf16((n_full, H, D), w.seed, f"full_{c}").to(dev) for c in "qkv")
+    if gpu_inputs:
+        qf, kf, vf = (gpu_randn_bf16((n_full, H, D), 1000 * w.seed + 100 + i, dev) for i in range(3))
+    else:
+        qf, kf, vf = (workloads.randn_bf16((n_full, H, D), w.seed, f"full_{c}").to(dev) for c in "qkv")
     o_f = torch.empty(n_full, H, D, dtype=torch.bfloat16, device=dev)
     for _ in range(2):
         rcb.full_attention(cu_full, qf, kf, vf, o_f, scale=scale)
@@ -572,6 +647,8 @@ def main(argv=None):
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end measurement")
     ap.add_argument("--no-full", action="store_true", help="skip the full-attention baseline")
     ap.add_argument("--no-cfg", action="store_true", help="skip the guided (positive + negative branch) step")
+    ap.add_argument("--no-sweep", action="store_true",
+                    help="skip the 1024^2 reference sweep (1-10 refs) and the ragged serving batch")
     args = ap.parse_args(argv)
     ws, rank, local = dist_env()
     if args.warmup < 3:
