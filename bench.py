@@ -269,6 +269,9 @@ def run_ours(args, ws, rank, local):
     cfg = None
     if w.name == "edit1024_5ref" and not args.no_cfg:
         cfg = time_cfg_pair(dev, stream, scale, t_step)
+    linear = None
+    if not args.no_linear and t_full == t_full:
+        linear = linear_accounting(w, dev, stream, t_pre, t_step, t_full)
     sweep = ragged = None
     if w.name == "edit1024_5ref" and not args.no_sweep:
         sweep = [time_step_workload(x, dev, stream, scale) for x in workloads.SWEEP_1024]
@@ -313,6 +316,7 @@ def run_ours(args, ws, rank, local):
             "algorithmic_bytes": 2 * (seg.live_rows * H * D * 2) * 2 + acc.cache_bytes(w.requests, H, D),
         },
         "cfg_pair": cfg,
+        "linear_accounting": linear,
         "reference_sweep": sweep,
         "ragged_batch": ragged,
         "e2e": e2e,
@@ -388,6 +392,56 @@ def time_step_workload(w, dev, stream, scale, with_full=True):
         out["full_tflops"] = acc.flops(acc.full_units(w.requests), H, D) / t_full / 1e12
         out["measured_40step"] = acc.measured_ratio(t_full, t_pre, t_step, T_STEPS)
     return out
+
+
+def linear_accounting(w, dev, stream, t_pre, t_step, t_full):
+    """Context only: the per-token linear work of one layer that caching also
+    removes (App. C, "What the interaction model omits"), timed with cuBLAS
+    (torch.matmul, bf16) on random weights, folded into a 40-step model of one
+    layer.  Assumed layer shape (the paper does not state it): hidden =
+    heads x head_dim, Q/K/V and output projections, a two-matrix FFN of width
+    4 x hidden."""
+    import torch
+
+    H, D = w.num_heads, w.head_dim
+    hid, ffn = H * D, 4 * H * D
+    S = sum(x.n_lt + x.n_x for x in w.requests)
+    R = sum(x.n_r for x in w.requests)
+    ST = sum(x.n_st for x in w.requests)
+    g = torch.Generator(device=dev)
+    g.manual_seed(7)
+    mk = lambda *shape: (torch.randn(shape, generator=g, device=dev) * 0.02).to(torch.bfloat16)  # noqa: E731
+    w_qkv, w_o, w_up, w_dn = mk(hid, 3 * hid), mk(hid, hid), mk(hid, ffn), mk(ffn, hid)
+
+    def t_linear(n):
+        x = mk(n, hid)
+        def run():
+            qkv = x @ w_qkv
+            o = qkv[:, :hid] @ w_o
+            h = torch.nn.functional.gelu(o @ w_up, approximate="tanh")
+            return h @ w_dn
+        for _ in range(2):
+            run()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(5):
+            run()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / 5e3
+
+    flops_tok = 2 * (4 * hid * hid + 2 * hid * ffn)
+    tl_live, tl_static, tl_all = t_linear(S), t_linear(ST + R), t_linear(S + R)
+    full = T_STEPS * (t_full + tl_all)
+    cached = t_pre + tl_static + T_STEPS * (t_step + tl_live)
+    return {
+        "assumed_layer": f"hidden {hid}, QKV + O projections, FFN {ffn} (not stated by the paper)",
+        "linear_gflop_per_token": flops_tok / 1e9,
+        "linear_ms": {"live_tokens": tl_live * 1e3, "static_tokens": tl_static * 1e3, "all_tokens": tl_all * 1e3},
+        "cublas_tflops": flops_tok * (S + R) / tl_all / 1e12,
+        "modelled_40step_with_linear": full / cached,
+        "note": "context only: one layer, attention times measured above, linear work timed with cuBLAS",
+    }
 
 
 def time_cfg_pair(dev, stream, scale, t_step_positive):
@@ -647,6 +701,7 @@ def main(argv=None):
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end measurement")
     ap.add_argument("--no-full", action="store_true", help="skip the full-attention baseline")
     ap.add_argument("--no-cfg", action="store_true", help="skip the guided (positive + negative branch) step")
+    ap.add_argument("--no-linear", action="store_true", help="skip the cuBLAS-timed linear-work accounting")
     ap.add_argument("--no-sweep", action="store_true",
                     help="skip the 1024^2 reference sweep (1-10 refs) and the ragged serving batch")
     args = ap.parse_args(argv)
