@@ -83,6 +83,23 @@ extern "C" {
  * request must have zero anchors.                                            */
 #define REFCACHE_MASK_ISOLATED 2
 
+/* Cache format flag, OR-ed into mask_mode of refcache_bytes/refcache_create.
+ * An explicitly approximate variant of the paper's exact cache (Sec. 3.3
+ * reuses the cached K/V exactly): the cached rows are stored as OCP FP8 E4M3
+ * codes with one fp32 scale per (128-row tile of one request, head):
+ *   amax = max |x| over the tile's rows and the head's 128 columns,
+ *   s = amax / 448, code = E4M3(x * (448 / amax)) (round to nearest even,
+ *   IEEE fp32 divide and multiply; code 0 and s = 0 when amax = 0).
+ * Layout of one layer (refcache_fp8_ptr): K codes [rows_pad, H, 128], V codes
+ * transposed per head [H, 128, rows_pad], scales float32 [rows_pad / 128, H, 4]
+ * = (s_K, s_V, log2 s_V, 1 / s_V) (the last two 0 when s_V = 0); each
+ * request's cached rows start on a 128-row boundary and pad rows hold code 0.  head_dim must be 128 and the tcgen05 kernel selected.
+ * step_attention then quantises each live query row per head the same way
+ * (one scale per row), attends the cached keys on E4M3 tensor-core MMAs with
+ * E4M3 softmax weights, and the live keys exactly as in the bf16 cache; the
+ * prefill (refcache_build's outputs) is unchanged.  Half the cache bytes. */
+#define REFCACHE_CACHE_FP8 0x100
+
 /* Kernel selection (refcache_set_kernel): the tcgen05/TMEM/TMA kernel is the
  * default; the mma.sync kernel is the recompiled legacy-tensor-core baseline. */
 #define REFCACHE_KERNEL_TCGEN05 0
@@ -116,8 +133,8 @@ typedef struct refcache refcache_t; /* opaque; owns the per-layer K/V slots */
 /*
  * Device bytes a cache needs for `num_layers` layers (Sec. 3.3: per layer the
  * R rows' K and V, bf16, [cache_rows, num_heads, head_dim] each, plus the
- * anchors' rows in REFCACHE_MASK_BEYOND_ALT), plus its small work tables.
- * Returns 0 for invalid arguments.
+ * anchors' rows in REFCACHE_MASK_BEYOND_ALT; with REFCACHE_CACHE_FP8 the E4M3
+ * layout above), plus its small work tables.  Returns 0 for invalid arguments.
  */
 REFCACHE_API size_t refcache_bytes(int num_layers, int mask_mode, const refcache_segments_t* seg);
 
@@ -145,8 +162,18 @@ REFCACHE_API void refcache_destroy(refcache_t* cache);
  * Device pointers of layer `layer`'s K and V slots, each a THD bf16 tensor of
  * *rows rows: request b's cached rows follow request b-1's.  Cached rows are
  * R (Eq. 2), or [ST; R] in REFCACHE_MASK_BEYOND_ALT.  Any output may be NULL.
+ * REFCACHE_ERR_UNSUPPORTED for an E4M3 cache.
  */
 REFCACHE_API int refcache_kv_ptr(refcache_t* cache, int layer, void** k_slot, void** v_slot, int64_t* rows);
+
+/*
+ * Device pointers of layer `layer` of an E4M3 cache (REFCACHE_CACHE_FP8): the
+ * K codes [rows_pad, H, 128] (uint8), the V codes [H, 128, rows_pad] (uint8)
+ * and the scales [rows_pad / 128, H, 4] (float32), owned by the cache.  Any
+ * output may be NULL.  REFCACHE_ERR_UNSUPPORTED for a bf16 cache.
+ */
+REFCACHE_API int refcache_fp8_ptr(refcache_t* cache, int layer, void** k8, void** vt8, void** scales,
+                                  int64_t* rows_pad);
 
 /* 1 if `layer` has been built, 0 if not, < 0 on error. */
 REFCACHE_API int refcache_layer_built(refcache_t* cache, int layer);
@@ -154,9 +181,9 @@ REFCACHE_API int refcache_layer_built(refcache_t* cache, int layer);
 /*
  * Number of kernels one refcache_build (call = 0) or step_attention (call = 1)
  * on this cache launches with the kernel family currently selected
- * (refcache_set_kernel): the attention kernel, the cache copy (build, when
- * there are cached rows) and the combine of split items (when the cache's
- * work list has any).  < 0 on error.
+ * (refcache_set_kernel): the attention kernel, the cache write (build, when
+ * there are cached rows: a copy, or the E4M3 quantisation) and the combine of
+ * split items (when the cache's work list has any).  < 0 on error.
  */
 REFCACHE_API int refcache_call_launches(refcache_t* cache, int call);
 
@@ -165,8 +192,9 @@ REFCACHE_API int refcache_call_launches(refcache_t* cache, int call);
  * Eq. cost-pre).  q_static/k_static/v_static: [cu_static[batch], H, d] bf16,
  * each request's [ST; R] rows.  Writes o_static (same shape) for every ST and
  * R row, lse_static if non-NULL, and copies the cached rows' K and V into the
- * layer's slots.  The result does not depend on any live input, and repeated
- * builds with the same inputs produce the same bytes.
+ * layer's slots (an E4M3 cache: quantises them).  The result does not depend
+ * on any live input, and repeated builds with the same inputs produce the
+ * same bytes.
  */
 REFCACHE_API int refcache_build(refcache_t* cache, int layer, const void* q_static, const void* k_static,
                    const void* v_static, void* o_static, float* lse_static, float softmax_scale,
@@ -178,7 +206,9 @@ REFCACHE_API int refcache_build(refcache_t* cache, int layer, const void* q_stat
  * v_live: [cu_live[batch], H, d] bf16, each request's [LT; X_t] rows.  Keys
  * are the request's own live rows followed by its cached rows of `layer`.
  * Writes o_live (same shape) and lse_live if non-NULL.
- * Returns REFCACHE_ERR_NOT_BUILT if the layer was never built.
+ * Returns REFCACHE_ERR_NOT_BUILT if the layer was never built, and
+ * REFCACHE_ERR_UNSUPPORTED for an E4M3 cache while the mma.sync kernel is
+ * selected.
  */
 REFCACHE_API int step_attention(refcache_t* cache, int layer, const void* q_live, const void* k_live,
                    const void* v_live, void* o_live, float* lse_live, float softmax_scale,

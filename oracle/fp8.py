@@ -176,7 +176,7 @@ def quantize_queries(q_bits):
     return codes, s
 
 
-def step_fp8(q_l, k_l, v_l, k_cache_deq, v_cache_deq, scale, pairs):
+def step_fp8(q_l, k_l, v_l, k_cache_deq, v_cache_deq, scale, pairs, bound=False):
     """One request's step over the quantised cache, for the (live row, head)
     pairs given: returns (out [P, d], lse [P]) in fp64.
 
@@ -185,6 +185,17 @@ def step_fp8(q_l, k_l, v_l, k_cache_deq, v_cache_deq, scale, pairs):
     per-row E4M3 block); one softmax over all of them with the scores scaled
     by ``scale``.  Every live row sees every key of its request (the mask of
     App. C's step for live rows, with the cache holding R or [ST; R]).
+
+    With ``bound``, also returns [P, d] worst-case bounds of what rounding
+    the softmax weights can add to each output (the CUDA path rounds the
+    weights of cached keys to E4M3 and those of live keys to bf16, and its
+    output to bf16).  With w_k = exp(s_k - max) and l = sum w_k: a weight
+    rounded to E4M3 is off by at most 2^-4 w_k in the normal range and by
+    half the subnormal step, 2^-10, below it (taken as 2^-9, so that the
+    kernel's per-tile shift of the weights by at most a factor two below the
+    first tile's V scale is covered); a bf16 weight by 2^-9 w_k; the bf16
+    output by 2^-8 |o| (half an ulp is 2^-9 relative, doubled for margin):
+        bound_c = (sum_cache (2^-4 w_k + 2^-9) |v_kc| + sum_live 2^-9 w_k |v_kc|) / l + 2^-8 |o_c|
     """
     qf = bf16_to_f32(q_l).astype(np.float64)
     kf = bf16_to_f32(k_l).astype(np.float64)
@@ -193,6 +204,8 @@ def step_fp8(q_l, k_l, v_l, k_cache_deq, v_cache_deq, scale, pairs):
     d = qf.shape[2]
     out = np.zeros((len(pairs), d))
     lse = np.zeros(len(pairs))
+    bnd = np.zeros((len(pairs), d))
+    n_live = kf.shape[0]
     for p, (i, h) in enumerate(pairs):
         s_live = kf[:, h, :] @ qf[i, h]
         if k_cache_deq.shape[0]:
@@ -208,4 +221,10 @@ def step_fp8(q_l, k_l, v_l, k_cache_deq, v_cache_deq, scale, pairs):
         den = w.sum()
         out[p] = (w @ vals) / den
         lse[p] = m + np.log(den)
+        if bound:
+            av = np.abs(vals)
+            bnd[p] = ((2.0 ** -4 * w[n_live:] + 2.0 ** -9) @ av[n_live:]
+                      + 2.0 ** -9 * w[:n_live] @ av[:n_live]) / den + 2.0 ** -8 * np.abs(out[p])
+    if bound:
+        return out, lse, bnd
     return out, lse

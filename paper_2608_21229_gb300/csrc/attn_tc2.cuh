@@ -60,6 +60,23 @@
 //                      group is full.
 //   stage_full[s]      the producers' TMA bytes of both CTAs (leader's barrier)
 //   q_full / q_empty   per Q buffer, once per item
+//
+// E4M3 cache (kF8): key range B is the quantised reference cache -- K as
+// E4M3 codes [rows_pad, H, 128] and V transposed per head [H, 128, rows_pad],
+// both K-major operands, with one fp32 scale (s_K, s_V) per 128-row tile and
+// head.  Its tiles run as kind::f8f6f4 MMAs (K = 32 per instruction, half
+// the tensor cycles of bf16); range A (the live rows) stays bf16.  At the
+// start of an item with cached tiles every softmax thread quantises its own
+// query row of this head into an E4M3 Q tile (one scale per row), and the
+// first cached tile's S waits for it (q8_full, one arrival per softmax warp
+// of both CTAs).  The
+// scales enter the softmax, so one O accumulator serves both ranges: with
+// s_ref = s_V of the item's first cached tile, the weights written are
+//   live tile:    exp2(u - m) / s_ref                   (bf16, u = scaled score)
+//   cached tile:  exp2(u + delta - m), delta = log2(s_V / s_ref)   (E4M3)
+// where the running maximum m is taken over u + delta, so E4M3 weights stay
+// at most 2^8; each tile adds its unshifted weight sum to l, and
+// O = s_ref * acc / l.
 #pragma once
 #include "attn_tc.cuh"
 
@@ -78,14 +95,20 @@ constexpr uint32_t kKBox = 64 * 128;        // one K box: 64 rows x 128 bytes
 constexpr int kWarpArrivals = 8;            // 4 softmax warps in each of the 2 CTAs
 constexpr int kProducerWarp = 4, kMmaWarp = 5, kGateWarp = 6;
 constexpr uint32_t kGateBarrier = 1;  // named barrier of the MMA and gate warps (0 is __syncthreads)
+constexpr uint32_t kKHalf8 = 64 * 128;   // 8 KB: this CTA's 64 keys x 128 d of an E4M3 K tile
+constexpr uint32_t kVHalf8 = 64 * 128;   // 8 KB: this CTA's 64 d x 128 keys of an E4M3 V^T tile
+constexpr uint32_t kQ8Tile = 128 * 128;  // this CTA's 128 query rows as E4M3
 static_assert(kStages == 4, "pair_done indexing assumes four stages");
 
-struct Smem {
+template <bool kF8>
+struct SmemT {
   static constexpr uint32_t kQ = 0;                // Q buffers 0 and 1 (this CTA's 128 rows)
   static constexpr uint32_t kRing = 2 * kQTile;    // stage s: [K half | V half]
-  static constexpr uint32_t kBars = kRing + kStages * kStage;
+  static constexpr uint32_t kQ8 = kRing + kStages * kStage;  // E4M3 Q tile (kF8 only)
+  static constexpr uint32_t kScales = kQ8 + (kF8 ? kQ8Tile : 0u);  // per softmax warp: 2 x 16 B (kF8 only)
+  static constexpr uint32_t kBars = kScales + (kF8 ? 4u * 32u : 0u);
   static constexpr int kQFull = 0, kQEmpty = 2, kStageFull = 4, kPairDone = 4 + kStages, kPFull = kPairDone + 4,
-                       kMmaDone = kPFull + 2, kNumBars = kMmaDone + 1;
+                       kMmaDone = kPFull + 2, kQ8Full = kMmaDone + 1, kNumBars = kQ8Full + 1;
   static constexpr uint32_t kTmemHolder = kBars + 8 * kNumBars;
   static constexpr uint32_t kAbort = kTmemHolder + 4;
   static constexpr uint32_t kUsed = kAbort + 4;
@@ -93,6 +116,7 @@ struct Smem {
   static constexpr uint32_t kDynamic = kUsed + 1024 < kMaxDynamic ? kUsed + 1024 : kMaxDynamic;
   static_assert(kUsed <= kMaxDynamic, "shared-memory layout too large");
 };
+using Smem = SmemT<false>;
 
 // Phase parity of pair_done[g % 4] / stage_full[g % 4] for group g.
 __device__ __forceinline__ uint32_t group_parity(int g) { return static_cast<uint32_t>(g >> 2) & 1u; }
@@ -118,6 +142,7 @@ __device__ __forceinline__ bool wait_cl_warp(uint32_t bar, uint32_t parity, cons
 }
 }  // namespace tc2
 
+template <bool kF8>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
     attn_tc2_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_ka,
                     const __grid_constant__ CUtensorMap tm_va, const __grid_constant__ CUtensorMap tm_kb,
@@ -133,10 +158,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
   using tc2::group_parity;
   using tc2::wait_cl;
   using tc2::wait_cl_warp;
-  using L = tc2::Smem;
+  using tc2::kKHalf8;
+  using tc2::kVHalf8;
+  using L = tc2::SmemT<kF8>;
   constexpr int D = tc2::kD;
   constexpr uint32_t kIdescS = idesc_bf16_f32(256, 128, false);
   constexpr uint32_t kIdescO = idesc_bf16_f32(256, D, true);
+  constexpr uint32_t kIdesc8 = idesc_e4m3_f32(256, 128);  // S and O of cached tiles (N = 128 keys or d)
 
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -169,6 +197,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
       mbar_init(bar(L::kPairDone + s), 1);
     }
     mbar_init(bar(L::kMmaDone), 1);
+    mbar_init(bar(L::kQ8Full), kWarpArrivals);
     *abort_flag = 0;
     fence_barrier_init();
     fence_proxy_async_smem();
@@ -204,7 +233,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         if (g >= kStages && !wait_one(bar(L::kPairDone + slot), group_parity(g - kStages), ctl, 2)) return false;
         const uint32_t dst = base + L::kRing + static_cast<uint32_t>(slot) * kStage;
         const uint32_t full = lbar(L::kStageFull + slot);
-        const uint32_t bytes = 2 * ((kj >= 0 ? kKHalf : 0u) + (vj >= 0 ? kVHalf : 0u));
+        const TileSrc ks = tile_src(tk, na, kj >= 0 ? kj : 0);
+        const TileSrc vs = tile_src(tk, na, vj >= 0 ? vj : 0);
+        const bool k8 = kF8 && kj >= 0 && ks.in_b, v8 = kF8 && vj >= 0 && vs.in_b;
+        const uint32_t bytes =
+            2 * ((kj >= 0 ? (k8 ? kKHalf8 : kKHalf) : 0u) + (vj >= 0 ? (v8 ? kVHalf8 : kVHalf) : 0u));
         if (skip_next) {  // fault injection: the leader never arms or loads this stage
           skip_next = false;
         } else {
@@ -212,16 +245,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
             mbar_arrive_expect_tx(bar(L::kStageFull + slot), bytes);
             armed_phase[slot] = static_cast<int>(group_parity(g));
           }
-          if (kj >= 0) {  // keys [64 r, 64 r + 64) of the tile, both head-dim boxes
-            const TileSrc src = tile_src(tk, na, kj);
-            const void* map = src.in_b ? &tm_kb : &tm_ka;
+          if (k8) {  // E4M3 keys [64 r, 64 r + 64): one box of 64 rows x 128 bytes
+            tma_load_2d_pair(dst, &tm_kb, full, head * D, ks.row + 64 * static_cast<int>(rank));
+          } else if (kj >= 0) {  // keys [64 r, 64 r + 64) of the tile, both head-dim boxes
+            const void* map = ks.in_b ? &tm_kb : &tm_ka;
             for (int ch = 0; ch < 2; ++ch)
-              tma_load_2d_pair(dst + ch * kKBox, map, full, head * D + ch * 64, src.row + 64 * static_cast<int>(rank));
+              tma_load_2d_pair(dst + ch * kKBox, map, full, head * D + ch * 64, ks.row + 64 * static_cast<int>(rank));
           }
-          if (vj >= 0) {  // head-dim columns [64 r, 64 r + 64) of all 128 keys
-            const TileSrc src = tile_src(tk, na, vj);
-            const void* map = src.in_b ? &tm_vb : &tm_va;
-            tma_load_2d_pair(dst + kKHalf, map, full, head * D + 64 * static_cast<int>(rank), src.row);
+          if (v8) {  // E4M3 V^T rows d in [64 r, 64 r + 64), all 128 keys
+            tma_load_2d_pair(dst + kKHalf, &tm_vb, full, vs.row, head * D + 64 * static_cast<int>(rank));
+          } else if (vj >= 0) {  // head-dim columns [64 r, 64 r + 64) of all 128 keys
+            const void* map = vs.in_b ? &tm_vb : &tm_va;
+            tma_load_2d_pair(dst + kKHalf, map, full, head * D + 64 * static_cast<int>(rank), vs.row);
           }
         }
         ++g;
@@ -267,6 +302,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
       const uint64_t kd0 = sdesc_sw128(base + L::kRing, 16, 1024);
       const uint64_t vd0 = sdesc_sw128(base + L::kRing + kKHalf, kBoxBytes, 1024);
       const uint64_t qdesc0 = sdesc_sw128(base + L::kQ, 16, 1024);
+      // E4M3 operands: Q8 (128 rows x 128 B), K8 half (64 rows x 128 B), V^T half (64 d x 128 B); a
+      // K = 32 step advances 32 bytes inside the swizzle atom
+      const uint64_t q8d = sdesc_sw128(base + L::kQ8, 16, 1024);
+      const uint64_t vd80 = sdesc_sw128(base + L::kRing + kKHalf, 16, 1024);
       // S step kk: A = Q (128-row boxes of 16 KB), B = this CTA's 64 keys (64-row boxes of 8 KB)
       auto q_off = [](int kk) -> uint64_t {
         return (static_cast<uint32_t>(kk >> 2) * kBoxBytes + static_cast<uint32_t>(kk & 3) * 32u) >> 4;
@@ -293,9 +332,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
               tc_fence_after();
               const uint64_t kd = kd0 + static_cast<uint64_t>(slot) * (kStage >> 4);
               const uint32_t d_s = tmem + kColS + (static_cast<uint32_t>((t0 + n) & 1) << 7);
+              if (kF8 && n >= na) {
 #pragma unroll
-              for (int kk = 0; kk < D / 16; ++kk)
-                tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
+                for (int kk = 0; kk < 4; ++kk)
+                  tc2_mma_ss_f8(d_s, q8d + ((32u * kk) >> 4), kd + ((32u * kk) >> 4), kIdesc8, kk > 0 ? 1u : 0u);
+              } else {
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk)
+                  tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
+              }
               if (n == nkv - 1) tc2_commit_mc(bar(L::kQEmpty + qb), 3);
             }
             tc2_commit_mc(bar(L::kPairDone + slot), 3);
@@ -315,15 +360,37 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
             const uint64_t vd = vd0 + soff;
             const uint32_t a_p = tmem + kColP + (static_cast<uint32_t>(t & 1) << 6);
             const uint32_t acc0 = j > 0 ? 1u : 0u;
+            const bool pv8 = kF8 && j >= na;      // P_j V_j on E4M3 operands
+            const bool s8 = kF8 && j + 2 >= na;   // S_j+2 on E4M3 operands
+            const uint64_t vd8 = vd80 + soff;
             if (j + 2 < nkv) {
               const uint64_t kd = kd0 + soff;
               const uint32_t d_s = tmem + kColS + (static_cast<uint32_t>(t & 1) << 7);
+              if (!s8) {
 #pragma unroll
-              for (int kk = 0; kk < 8; ++kk) {
-                tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, kk > 0 ? 1u : acc0);
-                tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
+                for (int kk = 0; kk < 8; ++kk) {
+                  tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, kk > 0 ? 1u : acc0);
+                  tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
+                }
+              } else if (pv8) {
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk) {
+                  tc2_mma_ts_f8(tmem + kColO, a_p + 8u * kk, vd8 + ((32u * kk) >> 4), kIdesc8, kk > 0 ? 1u : acc0);
+                  tc2_mma_ss_f8(d_s, q8d + ((32u * kk) >> 4), kd + ((32u * kk) >> 4), kIdesc8, kk > 0 ? 1u : 0u);
+                }
+              } else {  // the last live tiles' P.V beside the first cached tiles' S
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk) {
+                  tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, kk > 0 ? 1u : acc0);
+                  if (kk < 4)
+                    tc2_mma_ss_f8(d_s, q8d + ((32u * kk) >> 4), kd + ((32u * kk) >> 4), kIdesc8, kk > 0 ? 1u : 0u);
+                }
               }
               if (j + 2 == nkv - 1) tc2_commit_mc(bar(L::kQEmpty + qb), 3);
+            } else if (pv8) {
+#pragma unroll
+              for (int kk = 0; kk < 4; ++kk)
+                tc2_mma_ts_f8(tmem + kColO, a_p + 8u * kk, vd8 + ((32u * kk) >> 4), kIdesc8, kk > 0 ? 1u : acc0);
             } else {
 #pragma unroll
               for (int kk = 0; kk < 8; ++kk)
@@ -348,25 +415,31 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
     // The same group sequence as the MMA warp; every wait is bounded, and a
     // failed wait is passed on through the handshake, after which both leave.
     if (leader) {
-      int g = 0, t0 = 0, qi = 0;
+      int g = 0, t0 = 0, qi = 0, q8i = 0;
       for (int item = cluster; item < args.n_items; item += n_clusters) {
         Task tk;
         int head, na;
         decode_item(args, item, tk, head);
         const int nkv = n_key_tiles(tk, na);
         if (nkv == 0) continue;
+        // the first cached tile's S also needs the E4M3 Q tile of both CTAs
+        const bool q8 = kF8 && nkv > na;
+        const uint32_t q8_parity = static_cast<uint32_t>(q8i) & 1u;
         bool ok = wait_cl_warp(bar(L::kQFull + (qi & 1)), static_cast<uint32_t>(qi >> 1) & 1u, ctl, 3);
         for (int n = 0; n < 2; ++n, ++g) {
           ok = ok && wait_cl_warp(bar(L::kStageFull + (g & (kStages - 1))), group_parity(g), ctl, 4);
+          if (q8 && n == na) ok = ok && wait_cl_warp(bar(L::kQ8Full), q8_parity, ctl, 14);
           if (bar_red_or(tc2::kGateBarrier, 64, !ok)) goto gate_done;
         }
         for (int j = 0; j < nkv; ++j, ++g) {
           const int t = t0 + j;
           ok = wait_cl_warp(bar(L::kPFull + (t & 1)), static_cast<uint32_t>(t >> 1) & 1u, ctl, 7);
+          if (q8 && j + 2 == na) ok = ok && wait_cl_warp(bar(L::kQ8Full), q8_parity, ctl, 14);
           if (bar_red_or(tc2::kGateBarrier, 64, !ok)) goto gate_done;
         }
         t0 += nkv;
         ++qi;
+        if (q8) ++q8i;
       }
     gate_done:;
     }
@@ -401,9 +474,88 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         continue;
       }
       float m_run = 0.f, l_run = 0.f;
+      // E4M3 cache: this row's query scale (folded into sl2) and the weight scale s_ref
+      float c_row = sl2, s_ref = 1.f, l2_ref = 0.f;
+      const int scale_row0 = kF8 ? (tk.b_row0 >> 7) * args.num_heads + head : 0;
+      if (kF8 && nkv > na) {
+        // quantise this thread's query row of this head into the E4M3 Q tile:
+        // s = amax / 448, code = E4M3(x * (448 / amax)), round to nearest even
+        uint4 raw[16];
+        if (row_ok) {
+          const uint4* src = reinterpret_cast<const uint4*>(args.q + grow * args.row_stride + static_cast<int64_t>(head) * D);
+#pragma unroll
+          for (int c = 0; c < 16; ++c) raw[c] = src[c];
+        } else {
+#pragma unroll
+          for (int c = 0; c < 16; ++c) raw[c] = make_uint4(0, 0, 0, 0);
+        }
+        float amax = 0.f;
+#pragma unroll
+        for (int c = 0; c < 16; ++c) {
+          const uint32_t w4[4] = {raw[c].x, raw[c].y, raw[c].z, raw[c].w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e)
+            amax = fmax3(amax, fabsf(__uint_as_float(w4[e] << 16)), fabsf(__uint_as_float(w4[e] & 0xFFFF0000u)));
+        }
+        const float inv = amax > 0.f ? __fdiv_rn(448.f, amax) : 0.f;
+        const uint32_t q8_row = base + L::kQ8 + static_cast<uint32_t>(trow) * 128u;
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {  // 16 codes per 16-byte chunk, 128-byte swizzle
+          uint32_t w[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const uint32_t x0 = e < 2 ? (&raw[2 * c].x)[2 * e] : (&raw[2 * c + 1].x)[2 * e - 4];
+            const uint32_t x1 = e < 2 ? (&raw[2 * c].x)[2 * e + 1] : (&raw[2 * c + 1].x)[2 * e - 3];
+            w[e] = pack_e4m3x4(__fmul_rn(__uint_as_float(x0 << 16), inv), __fmul_rn(__uint_as_float(x0 & 0xFFFF0000u), inv),
+                               __fmul_rn(__uint_as_float(x1 << 16), inv), __fmul_rn(__uint_as_float(x1 & 0xFFFF0000u), inv));
+          }
+          st_shared_v4(q8_row + ((static_cast<uint32_t>(c) ^ static_cast<uint32_t>(trow & 7)) << 4),
+                       make_uint4(w[0], w[1], w[2], w[3]));
+        }
+        // visible to the tensor core, then one arrival per warp of both CTAs
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_release_cluster(mapa_shared(bar(L::kQ8Full), 0));
+        c_row = sl2 * __fdiv_rn(amax, 448.f);
+        const float4 sc0 = args.b_scales[scale_row0];
+        s_ref = sc0.y > 0.f ? sc0.y : 1.f;
+        l2_ref = sc0.y > 0.f ? sc0.z : 0.f;
+      }
+      // the scales of cached tiles are fetched one tile ahead by asynchronous
+      // copies into this warp's two slots (an ordinary load still in flight
+      // would hold up the release of the next P arrival)
+      const uint32_t sc_slots = base + L::kScales + static_cast<uint32_t>(warp) * 32u;
+      if (kF8 && na < nkv) {
+        if (lane == 0) cp_async_16(sc_slots, args.b_scales + scale_row0);
+        cp_async_commit();
+      }
       for (int j = 0; j < nkv; ++j, ++t) {
         const int b = t & 1;
         const TileSrc src = tile_src(tk, na, j);
+        // per-tile constants: u = c * s + shift is the shifted scaled score, the
+        // weight written is exp2(u - m + wshift), the tile adds lscale * sum to l
+        const bool t8 = kF8 && j >= na;
+        float c_t = sl2, shift = 0.f, wshift = -l2_ref, lscale = s_ref;
+        if (t8) {
+          const int jb = j - na;  // index among the item's cached tiles
+          if (j + 1 < nkv) {
+            if (lane == 0)
+              cp_async_16(sc_slots + 16u * static_cast<uint32_t>((jb + 1) & 1),
+                          args.b_scales + scale_row0 + (jb + 1) * args.num_heads);
+            cp_async_commit();
+            cp_async_wait<1>();
+          } else {
+            cp_async_wait<0>();
+          }
+          __syncwarp();
+          const float4 sc = ld_shared_f4(sc_slots + 16u * static_cast<uint32_t>(jb & 1));
+          c_t = fmaxf(c_row * sc.x, 1e-30f);
+          // delta = log2(s_V / s_ref); an all-zero V tile (s_V = 0) takes delta = 0
+          const bool nz = sc.y > 0.f;
+          shift = nz ? sc.z - l2_ref : 0.f;
+          wshift = 0.f;
+          lscale = nz ? s_ref * sc.w : 1.f;  // 2^-delta
+        }
         // S_j is ready and P buffer b is free once group G + j is complete
         if (!wait_group(G + j, 8)) goto softmax_done;
         tc_fence_after();
@@ -441,7 +593,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
           for (int c = 3; c < 31; c += 2) mx[k] = fmax3(mx[k], s[32 * k + c], s[32 * k + c + 1]);
           mx[k] = fmaxf(mx[k], s[32 * k + 31]);
         }
-        const float m_tile = fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3])) * sl2;
+        const float m_tile = fmaf(fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3])), c_t, shift);
         if (j == 0) {
           m_run = m_tile;
         } else if (__any_sync(0xffffffffu, m_tile > m_run + 8.0f)) {
@@ -470,31 +622,54 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
             tmem_st16(t_o + 16u * cc, o);
           }
         }
-        // P = exp2(scale * S - m) as bf16 pairs into P buffer b, 32 keys (16 columns) at a time
-        const f32x2 negm = make_f32x2(-m_run, -m_run);
+        // P = exp2(c * S + shift - m) into P buffer b: bf16 pairs (32 keys = 16
+        // columns at a time), or for a cached tile E4M3 quads (32 keys = 8 columns)
+        const float bias = (kF8 ? shift + wshift : 0.f) - m_run;
+        const f32x2 negm = make_f32x2(bias, bias);
+        const f32x2 c2 = kF8 ? make_f32x2(c_t, c_t) : sl2x2;
         const uint32_t t_p = tmem + lane_off + kColP + 64u * b;
         f32x2 lacc[4];
 #pragma unroll
         for (int i = 0; i < 4; ++i) lacc[i] = make_f32x2(0.f, 0.f);
+        if (t8) {
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          uint32_t pk[16];
+          for (int k = 0; k < 4; ++k) {
+            uint32_t pk[8];
 #pragma unroll
-          for (int c = 0; c < 16; ++c) {
-            const f32x2 e = fma_f32x2(make_f32x2(s[32 * k + 2 * c], s[32 * k + 2 * c + 1]), sl2x2, negm);
-            float e0, e1;
-            split_f32x2(e, e0, e1);
-            const float x = ex2_approx(e0), y = ex2_approx(e1);
-            lacc[c & 3] = add_f32x2(lacc[c & 3], make_f32x2(x, y));
-            pk[c] = pack_bf16x2(x, y);
+            for (int c = 0; c < 8; ++c) {
+              const f32x2 e01 = fma_f32x2(make_f32x2(s[32 * k + 4 * c], s[32 * k + 4 * c + 1]), c2, negm);
+              const f32x2 e23 = fma_f32x2(make_f32x2(s[32 * k + 4 * c + 2], s[32 * k + 4 * c + 3]), c2, negm);
+              float e0, e1, e2, e3;
+              split_f32x2(e01, e0, e1);
+              split_f32x2(e23, e2, e3);
+              const float x0 = ex2_approx(e0), x1 = ex2_approx(e1), x2 = ex2_approx(e2), x3 = ex2_approx(e3);
+              lacc[(2 * c) & 3] = add_f32x2(lacc[(2 * c) & 3], make_f32x2(x0, x1));
+              lacc[(2 * c + 1) & 3] = add_f32x2(lacc[(2 * c + 1) & 3], make_f32x2(x2, x3));
+              pk[c] = pack_e4m3x4(x0, x1, x2, x3);
+            }
+            tmem_st8(t_p + 8u * k, pk);
           }
-          tmem_st16(t_p + 16u * k, pk);
+        } else {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            uint32_t pk[16];
+#pragma unroll
+            for (int c = 0; c < 16; ++c) {
+              const f32x2 e = fma_f32x2(make_f32x2(s[32 * k + 2 * c], s[32 * k + 2 * c + 1]), c2, negm);
+              float e0, e1;
+              split_f32x2(e, e0, e1);
+              const float x = ex2_approx(e0), y = ex2_approx(e1);
+              lacc[c & 3] = add_f32x2(lacc[c & 3], make_f32x2(x, y));
+              pk[c] = pack_bf16x2(x, y);
+            }
+            tmem_st16(t_p + 16u * k, pk);
+          }
         }
         {
           const f32x2 l2 = add_f32x2(add_f32x2(lacc[0], lacc[1]), add_f32x2(lacc[2], lacc[3]));
           float lo, hi;
           split_f32x2(l2, lo, hi);
-          l_run += lo + hi;
+          l_run += kF8 ? (lo + hi) * lscale : lo + hi;
         }
         // the MMA thread waits only for P: the leader's warp 0 first makes
         // sure that the stage of P_j V_j's group (G + j + 2) has landed
@@ -509,7 +684,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
       {
         if (!wait_group(G + nkv + 1, 10)) goto softmax_done;  // the item's last group
         tc_fence_after();
-        const float inv_l = 1.0f / l_run;
+        const float inv_l = kF8 ? s_ref / l_run : 1.0f / l_run;
         const uint32_t t_o = tmem + lane_off + kColO;
         if (tk.part > 0) {
           // a part of a split item: O / l in fp32 and m + log l to its workspace slot

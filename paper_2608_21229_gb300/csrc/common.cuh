@@ -48,6 +48,7 @@ struct AttnArgs {
   float* part_o;                // workspace of partial results: [slot][rows_per_task][D] fp32, O / l
   float* part_lse;              //                               [slot][rows_per_task] fp32, m + log l
   uint64_t timeout_ns;          // bound of every in-kernel wait
+  const float4* b_scales;       // E4M3 key range B: (s_K, s_V, log2 s_V, 1/s_V) per (128-row tile, head), tile-major
   // raw pointers, used by the mma.sync kernel (the tcgen05 kernel reads
   // through tensor maps)
   const __nv_bfloat16* q;

@@ -20,10 +20,12 @@
 #include "attn_tc.cuh"
 #include "attn_tc2.cuh"
 #include "attn_combine.cuh"
+#include "cache_fp8.cuh"
 
 using rc::AttnArgs;
 using rc::CombineJob;
 using rc::CopySeg;
+using rc::QuantTile;
 using rc::Task;
 
 namespace {
@@ -53,8 +55,8 @@ struct DeviceInfo {
   bool checked = false;
   bool ok = false;
   int num_sms = 0;
-  bool attr_set[5] = {false, false, false, false, false};
-  int max_clusters = 0;
+  bool attr_set[6] = {false, false, false, false, false, false};
+  int max_clusters[2] = {0, 0};  // CTA pairs of attn_tc2_kernel<false>, <true> that fit at once
 };
 DeviceInfo g_dev[kMaxDevices];
 std::mutex g_dev_mu;
@@ -119,6 +121,22 @@ int make_tmap(CUtensorMap* m, const void* base, int64_t rows, int H, int D, uint
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return fail(REFCACHE_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
+  return REFCACHE_OK;
+}
+
+// Byte matrix (E4M3 codes) of `outer` rows x `inner` bytes, row pitch `inner`;
+// box = 128 bytes x 64 rows with the 128-byte swizzle.
+int make_tmap_u8(CUtensorMap* m, const void* base, int64_t inner, int64_t outer) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return fail(REFCACHE_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(std::max<int64_t>(outer, 1))};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(inner)};
+  const cuuint32_t box[2] = {128, 64};
+  const cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(REFCACHE_ERR_CUDA, "cuTensorMapEncodeTiled (u8) failed (%d)", static_cast<int>(r));
   return REFCACHE_OK;
 }
 
@@ -192,35 +210,41 @@ int launch_tc(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info,
   return REFCACHE_OK;
 }
 
-// CTA pairs of the head-dim-128 kernel that run at once on this device (the
-// persistent grid); sets the kernel's shared-memory attribute on first use.
+// CTA pairs of the head-dim-128 kernel (bf16 key range B, or E4M3 with kF8)
+// that run at once on this device (the persistent grid); sets the kernel's
+// shared-memory attribute on first use.
+template <bool kF8>
 int tc2_clusters(DeviceInfo* info, int* clusters_out) {
-  constexpr uint32_t smem = rc::tc2::Smem::kDynamic;
-  if (!info->attr_set[4]) {
-    cudaError_t e = cudaFuncSetAttribute(rc::attn_tc2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  constexpr uint32_t smem = rc::tc2::SmemT<kF8>::kDynamic;
+  const int key = kF8 ? 5 : 4;
+  if (!info->attr_set[key]) {
+    cudaError_t e =
+        cudaFuncSetAttribute(rc::attn_tc2_kernel<kF8>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_tc2_kernel)");
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3(2 * static_cast<unsigned>(info->num_sms / 2), 1, 1);
     cfg.blockDim = dim3(rc::tc2::kThreads, 1, 1);
     cfg.dynamicSmemBytes = smem;
     int clusters = 0;
-    e = cudaOccupancyMaxActiveClusters(&clusters, rc::attn_tc2_kernel, &cfg);
+    e = cudaOccupancyMaxActiveClusters(&clusters, rc::attn_tc2_kernel<kF8>, &cfg);
     if (e != cudaSuccess || clusters < 1) clusters = info->num_sms / 2;
-    info->max_clusters = clusters;
-    info->attr_set[4] = true;
+    info->max_clusters[kF8 ? 1 : 0] = clusters;
+    info->attr_set[key] = true;
   }
-  *clusters_out = info->max_clusters;
+  *clusters_out = info->max_clusters[kF8 ? 1 : 0];
   return REFCACHE_OK;
 }
 
 // The CTA-pair kernel (head_dim 128): grid = 2 x the clusters that fit at once.
+template <bool kF8>
 int launch_tc2(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info, cudaStream_t s) {
-  constexpr uint32_t smem = rc::tc2::Smem::kDynamic;
+  constexpr uint32_t smem = rc::tc2::SmemT<kF8>::kDynamic;
   int max_clusters = 0;
-  int rc = tc2_clusters(info, &max_clusters);
+  int rc = tc2_clusters<kF8>(info, &max_clusters);
   if (rc) return rc;
   const int clusters = std::min(a.n_items, max_clusters);
-  rc::attn_tc2_kernel<<<2 * clusters, rc::tc2::kThreads, smem, s>>>(maps[0], maps[1], maps[2], maps[3], maps[4], a);
+  rc::attn_tc2_kernel<kF8>
+      <<<2 * clusters, rc::tc2::kThreads, smem, s>>>(maps[0], maps[1], maps[2], maps[3], maps[4], a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "attn_tc2_kernel launch");
   return REFCACHE_OK;
@@ -252,6 +276,15 @@ struct Operands {
   float* lse;
 };
 
+// Key range B as an E4M3 cache (cache_fp8.cuh): codes of K [rows_pad, H, 128],
+// of V transposed [H, 128, rows_pad], and the scales of every tile and head.
+struct Fp8B {
+  const void* k8 = nullptr;
+  const void* vt8 = nullptr;
+  const float4* scales = nullptr;
+  int64_t rows_pad = 0;
+};
+
 // A per-item work list with split items (head-dim-128 tcgen05 kernel only):
 // the items, the combine jobs of the split ones and their workspace.
 struct ItemList {
@@ -264,7 +297,7 @@ struct ItemList {
 };
 
 int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands& op, float scale, DeviceInfo* info,
-                  cudaStream_t s, const ItemList* il = nullptr) {
+                  cudaStream_t s, const ItemList* il = nullptr, const Fp8B* f8 = nullptr) {
   if (n_tasks == 0) return REFCACHE_OK;
   AttnArgs a{};
   a.tasks = d_tasks;
@@ -283,8 +316,10 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
   a.kb = static_cast<const __nv_bfloat16*>(op.kb ? op.kb : op.ka);
   a.vb = static_cast<const __nv_bfloat16*>(op.vb ? op.vb : op.va);
   if (static_cast<int64_t>(n_tasks) * H > (1ll << 30)) return fail(REFCACHE_ERR_INVALID_ARG, "too many work items");
-  if (g_kernel.load() == REFCACHE_KERNEL_MMA_SYNC)
+  if (g_kernel.load() == REFCACHE_KERNEL_MMA_SYNC) {
+    if (f8) return fail(REFCACHE_ERR_UNSUPPORTED, "the E4M3 cache runs on the tcgen05 kernel only");
     return D == 64 ? launch_mma<64>(a, info, s) : launch_mma<128>(a, info, s);
+  }
   // K tiles of the CTA-pair kernel are loaded as two 64-row halves
   const uint32_t k_rows = D == 128 ? 64 : 128;
   CUtensorMap maps[5];
@@ -292,7 +327,11 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
   if ((rc = make_tmap(&maps[0], op.q, op.q_rows, H, D)) != 0) return rc;
   if ((rc = make_tmap(&maps[1], op.ka, op.a_rows, H, D, k_rows)) != 0) return rc;
   if ((rc = make_tmap(&maps[2], op.va, op.a_rows, H, D)) != 0) return rc;
-  if (op.kb && op.b_rows > 0) {
+  if (f8) {
+    if ((rc = make_tmap_u8(&maps[3], f8->k8, static_cast<int64_t>(H) * D, f8->rows_pad)) != 0) return rc;
+    if ((rc = make_tmap_u8(&maps[4], f8->vt8, f8->rows_pad, static_cast<int64_t>(H) * D)) != 0) return rc;
+    a.b_scales = f8->scales;
+  } else if (op.kb && op.b_rows > 0) {
     if ((rc = make_tmap(&maps[3], op.kb, op.b_rows, H, D, k_rows)) != 0) return rc;
     if ((rc = make_tmap(&maps[4], op.vb, op.b_rows, H, D)) != 0) return rc;
   } else {
@@ -308,7 +347,7 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
     a.part_o = il->part_o;
     a.part_lse = il->part_lse;
   }
-  if ((rc = launch_tc2(maps, a, info, s)) != 0) return rc;
+  if ((rc = f8 ? launch_tc2<true>(maps, a, info, s) : launch_tc2<false>(maps, a, info, s)) != 0) return rc;
   if (il && il->n_jobs > 0) {
     const dim3 grid(static_cast<unsigned>((a.rows_per_task + 7) / 8), static_cast<unsigned>(il->n_jobs));
     rc::combine_parts_kernel<128><<<grid, 256, 0, s>>>(il->jobs, il->part_o, il->part_lse, a.rows_per_task, a.out,
@@ -418,15 +457,32 @@ struct refcache {
   ItemList build_items, step_items;
   __nv_bfloat16* slots = nullptr;
   int64_t slot_elems = 0;
+  // E4M3 cache (REFCACHE_CACHE_FP8): per layer [k8 | vt8 | scales] of
+  // fp8_layer_bytes at slots8; each request's cached rows padded to 128
+  bool f8 = false;
+  int64_t rows_pad = 0;
+  QuantTile* d_qtiles = nullptr;
+  int n_qtiles = 0;
+  uint8_t* slots8 = nullptr;
+  size_t fp8_layer_bytes = 0;
   std::vector<char> built;
 };
 
 namespace {
 
-int cache_plan(int num_layers, int mode, const refcache_segments_t* seg, refcache* h, std::vector<Task>* build_tasks,
-               std::vector<Task>* step_tasks, std::vector<CopySeg>* copies, size_t* total_bytes) {
+// Bytes of one layer of an E4M3 cache: codes of K and V^T, and the scales.
+size_t fp8_layer_bytes(int64_t rows_pad, int H, int D) {
+  return align_up(static_cast<size_t>(rows_pad) * H * D, 256) * 2 +
+         align_up(static_cast<size_t>(rows_pad / 128) * H * sizeof(float4), 256);
+}
+
+int cache_plan(int num_layers, int mode_flags, const refcache_segments_t* seg, refcache* h,
+               std::vector<Task>* build_tasks, std::vector<Task>* step_tasks, std::vector<CopySeg>* copies,
+               std::vector<QuantTile>* qtiles, size_t* total_bytes) {
   if (!seg) return fail(REFCACHE_ERR_INVALID_ARG, "seg is NULL");
   if (num_layers < 1) return fail(REFCACHE_ERR_INVALID_ARG, "num_layers must be >= 1");
+  const bool f8 = (mode_flags & REFCACHE_CACHE_FP8) != 0;
+  const int mode = mode_flags & ~REFCACHE_CACHE_FP8;
   if (mode != REFCACHE_MASK_BEYOND && mode != REFCACHE_MASK_BEYOND_ALT && mode != REFCACHE_MASK_ISOLATED)
     return fail(REFCACHE_ERR_INVALID_ARG, "unknown mask_mode %d", mode);
   int rc;
@@ -453,13 +509,28 @@ int cache_plan(int num_layers, int mode, const refcache_segments_t* seg, refcach
   }
   if (cache_off[B] > max_rows) return fail(REFCACHE_ERR_INVALID_ARG, "cache rows too large");
   const int H = seg->num_heads, D = seg->head_dim;
+  if (f8 && D != 128) return fail(REFCACHE_ERR_UNSUPPORTED, "the E4M3 cache needs head_dim 128 (got %d)", D);
+  // E4M3 cache: request b's cached rows start at off8[b], a multiple of 128
+  std::vector<int64_t> off8(B + 1, 0);
+  std::vector<QuantTile> qt;
+  for (int b = 0; b < B; ++b) {
+    const int64_t nc = cache_off[b + 1] - cache_off[b];
+    off8[b + 1] = off8[b] + (nc + 127) / 128 * 128;
+    if (f8) {
+      const int src0 = mode == REFCACHE_MASK_BEYOND_ALT ? seg->cu_static[b] : seg->cu_static[b] + seg->n_anchor[b];
+      for (int64_t r = 0; r < nc; r += 128)
+        qt.push_back(QuantTile{static_cast<int32_t>(src0 + r), static_cast<int32_t>(std::min<int64_t>(128, nc - r)),
+                               static_cast<int32_t>(off8[b] + r), 0});
+    }
+  }
+  if (off8[B] > max_rows) return fail(REFCACHE_ERR_INVALID_ARG, "cache rows too large");
   const int tr = task_rows(D);
   std::vector<Task> bt, st;
   std::vector<CopySeg> cp;
   for (int b = 0; b < B; ++b) {
     const int s0 = seg->cu_static[b], ns = seg->cu_static[b + 1] - s0, na = seg->n_anchor[b];
     const int l0 = seg->cu_live[b], nl = seg->cu_live[b + 1] - l0;
-    const int c0 = static_cast<int>(cache_off[b]), nc = static_cast<int>(cache_off[b + 1] - cache_off[b]);
+    const int c0 = static_cast<int>(f8 ? off8[b] : cache_off[b]), nc = static_cast<int>(cache_off[b + 1] - cache_off[b]);
     if (mode == REFCACHE_MASK_BEYOND_ALT) {
       add_rows(bt, tr, s0, na, s0, na, 0, 0);            // anchor rows attend anchors only
       add_rows(bt, tr, s0 + na, ns - na, s0, ns, 0, 0);  // reference rows attend [ST; R]
@@ -467,7 +538,7 @@ int cache_plan(int num_layers, int mode, const refcache_segments_t* seg, refcach
       add_rows(bt, tr, s0, ns, s0, ns, 0, 0);  // [ST; R] rows attend [ST; R] (R only when isolated)
     }
     add_rows(st, tr, l0, nl, l0, nl, c0, nc);  // live rows attend their own rows, then the cache
-    if (nc > 0) {
+    if (nc > 0 && !f8) {
       CopySeg c{};
       c.src_row0 = mode == REFCACHE_MASK_BEYOND_ALT ? s0 : s0 + na;
       c.dst_row0 = c0;
@@ -482,8 +553,14 @@ int cache_plan(int num_layers, int mode, const refcache_segments_t* seg, refcach
   off = align_up(off + bt.size() * sizeof(Task), 256);
   off = align_up(off + st.size() * sizeof(Task), 256);
   off = align_up(off + cp.size() * sizeof(CopySeg), 256);
-  const size_t total = off + static_cast<size_t>(num_layers) * 2 * slot_elems * sizeof(__nv_bfloat16);
+  off = align_up(off + qt.size() * sizeof(QuantTile), 256);
+  const size_t layer_bytes = f8 ? fp8_layer_bytes(off8[B], H, D) : 2 * slot_elems * sizeof(__nv_bfloat16);
+  const size_t total = off + static_cast<size_t>(num_layers) * layer_bytes;
   if (h) {
+    h->f8 = f8;
+    h->rows_pad = off8[B];
+    h->n_qtiles = static_cast<int>(qt.size());
+    h->fp8_layer_bytes = f8 ? layer_bytes : 0;
     h->num_layers = num_layers;
     h->mode = mode;
     h->batch = B;
@@ -504,6 +581,7 @@ int cache_plan(int num_layers, int mode, const refcache_segments_t* seg, refcach
   if (build_tasks) *build_tasks = std::move(bt);
   if (step_tasks) *step_tasks = std::move(st);
   if (copies) *copies = std::move(cp);
+  if (qtiles) *qtiles = std::move(qt);
   *total_bytes = total;
   return REFCACHE_OK;
 }
@@ -529,13 +607,15 @@ int check_ptrs(std::initializer_list<const void*> ps, int64_t rows, const char* 
 // caller-sized cache memory is not touched).
 int plan_split_items(refcache* h, DeviceInfo* info, const std::vector<Task>& bt, const std::vector<Task>& st) {
   int clusters = 0;
-  int rc = tc2_clusters(info, &clusters);
+  int rc = tc2_clusters<false>(info, &clusters);
   if (rc) return rc;
+  int clusters_step = clusters;
+  if (h->f8 && h->rows_pad > 0 && (rc = tc2_clusters<true>(info, &clusters_step)) != 0) return rc;
   std::vector<Task> bi, si;
   std::vector<CombineJob> bj, sj;
   int bparts = 0, sparts = 0;
   plan_items(bt, h->H, clusters, &bi, &bj, &bparts);
-  plan_items(st, h->H, clusters, &si, &sj, &sparts);
+  plan_items(st, h->H, clusters_step, &si, &sj, &sparts);
   const int parts = std::max(bparts, sparts);  // build and step calls are stream-ordered: one workspace
   const int rows = task_rows(h->D);
   size_t off = 0;
@@ -591,7 +671,7 @@ extern "C" {
 
 size_t refcache_bytes(int num_layers, int mask_mode, const refcache_segments_t* seg) {
   size_t total = 0;
-  if (cache_plan(num_layers, mask_mode, seg, nullptr, nullptr, nullptr, nullptr, &total) != 0) return 0;
+  if (cache_plan(num_layers, mask_mode, seg, nullptr, nullptr, nullptr, nullptr, nullptr, &total) != 0) return 0;
   return total;
 }
 
@@ -601,8 +681,9 @@ int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refca
   refcache* h = new refcache();
   std::vector<Task> bt, st;
   std::vector<CopySeg> cp;
+  std::vector<QuantTile> qt;
   size_t total = 0;
-  int rc = cache_plan(num_layers, mask_mode, seg, h, &bt, &st, &cp, &total);
+  int rc = cache_plan(num_layers, mask_mode, seg, h, &bt, &st, &cp, &qt, &total);
   if (rc) {
     delete h;
     return rc;
@@ -639,11 +720,16 @@ int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refca
   off = align_up(off + st.size() * sizeof(Task), 256);
   h->d_copy = reinterpret_cast<CopySeg*>(h->mem + off);
   off = align_up(off + cp.size() * sizeof(CopySeg), 256);
+  h->d_qtiles = reinterpret_cast<QuantTile*>(h->mem + off);
+  off = align_up(off + qt.size() * sizeof(QuantTile), 256);
   h->slots = reinterpret_cast<__nv_bfloat16*>(h->mem + off);
+  h->slots8 = h->mem + off;
   cudaError_t e = cudaSuccess;
   if (!bt.empty() && e == cudaSuccess) e = cudaMemcpy(h->d_build, bt.data(), bt.size() * sizeof(Task), cudaMemcpyHostToDevice);
   if (!st.empty() && e == cudaSuccess) e = cudaMemcpy(h->d_step, st.data(), st.size() * sizeof(Task), cudaMemcpyHostToDevice);
   if (!cp.empty() && e == cudaSuccess) e = cudaMemcpy(h->d_copy, cp.data(), cp.size() * sizeof(CopySeg), cudaMemcpyHostToDevice);
+  if (!qt.empty() && e == cudaSuccess)
+    e = cudaMemcpy(h->d_qtiles, qt.data(), qt.size() * sizeof(QuantTile), cudaMemcpyHostToDevice);
   if (e != cudaSuccess) {
     if (h->owns) cudaFree(h->mem);
     delete h;
@@ -676,6 +762,7 @@ void refcache_destroy(refcache_t* h) {
 int refcache_kv_ptr(refcache_t* h, int layer, void** k_slot, void** v_slot, int64_t* rows) {
   int rc = check_handle_layer(h, layer);
   if (rc) return rc;
+  if (h->f8) return fail(REFCACHE_ERR_UNSUPPORTED, "an E4M3 cache has no bf16 slots (see refcache_fp8_ptr)");
   __nv_bfloat16* k = h->slots + static_cast<int64_t>(layer) * 2 * h->slot_elems;
   if (k_slot) *k_slot = k;
   if (v_slot) *v_slot = k + h->slot_elems;
@@ -683,14 +770,28 @@ int refcache_kv_ptr(refcache_t* h, int layer, void** k_slot, void** v_slot, int6
   return REFCACHE_OK;
 }
 
+int refcache_fp8_ptr(refcache_t* h, int layer, void** k8, void** vt8, void** scales, int64_t* rows_pad) {
+  int rc = check_handle_layer(h, layer);
+  if (rc) return rc;
+  if (!h->f8) return fail(REFCACHE_ERR_UNSUPPORTED, "not an E4M3 cache (create it with REFCACHE_CACHE_FP8)");
+  uint8_t* base = h->slots8 + static_cast<size_t>(layer) * h->fp8_layer_bytes;
+  const size_t codes = align_up(static_cast<size_t>(h->rows_pad) * h->H * h->D, 256);
+  if (k8) *k8 = base;
+  if (vt8) *vt8 = base + codes;
+  if (scales) *scales = base + 2 * codes;
+  if (rows_pad) *rows_pad = h->rows_pad;
+  return REFCACHE_OK;
+}
+
 int refcache_call_launches(refcache_t* h, int call) {
   if (!h) return fail(REFCACHE_ERR_INVALID_ARG, "cache is NULL");
   if (call != 0 && call != 1) return fail(REFCACHE_ERR_INVALID_ARG, "call must be 0 (build) or 1 (step)");
   const int n_tasks = call == 0 ? h->n_build : h->n_step;
-  if (n_tasks == 0) return call == 0 && h->n_copy > 0 ? 1 : 0;
+  const int cache_write = call == 0 && (h->n_copy > 0 || h->n_qtiles > 0) ? 1 : 0;
+  if (n_tasks == 0) return cache_write;
   const ItemList& il = call == 0 ? h->build_items : h->step_items;
   const bool tc = g_kernel.load() == REFCACHE_KERNEL_TCGEN05;
-  return (call == 0 && h->n_copy > 0 ? 1 : 0) + 1 + (tc && il.items && il.n_jobs > 0 ? 1 : 0);
+  return cache_write + 1 + (tc && il.items && il.n_jobs > 0 ? 1 : 0);
 }
 
 int refcache_layer_built(refcache_t* h, int layer) {
@@ -708,8 +809,17 @@ int refcache_build(refcache_t* h, int layer, const void* q_static, const void* k
   DeviceInfo* info = nullptr;
   if ((rc = enter_device(h, &info)) != 0) return rc;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (h->f8 && h->n_qtiles > 0) {
+    void *k8 = nullptr, *vt8 = nullptr, *sc = nullptr;
+    refcache_fp8_ptr(h, layer, &k8, &vt8, &sc, nullptr);
+    rc::quantize_cache_kernel<<<dim3(static_cast<unsigned>(h->n_qtiles), static_cast<unsigned>(h->H)), 256, 0, s>>>(
+        h->d_qtiles, static_cast<const uint4*>(k_static), static_cast<const uint4*>(v_static),
+        static_cast<uint8_t*>(k8), static_cast<uint8_t*>(vt8), static_cast<float4*>(sc), h->H, h->rows_pad);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "quantize_cache_kernel launch");
+  }
   void *kslot = nullptr, *vslot = nullptr;
-  refcache_kv_ptr(h, layer, &kslot, &vslot, nullptr);
+  if (!h->f8) refcache_kv_ptr(h, layer, &kslot, &vslot, nullptr);
   if (h->n_copy > 0) {
     const int row_u4 = h->H * h->D * 2 / 16;
     dim3 grid(static_cast<unsigned>(std::min<int64_t>(1024, (h->cache_rows * row_u4 + 255) / 256 / h->n_copy + 1)),
@@ -738,10 +848,19 @@ int step_attention(refcache_t* h, int layer, const void* q_live, const void* k_l
   DeviceInfo* info = nullptr;
   if ((rc = enter_device(h, &info)) != 0) return rc;
   void *kslot = nullptr, *vslot = nullptr;
-  refcache_kv_ptr(h, layer, &kslot, &vslot, nullptr);
+  Fp8B f8;
+  // an E4M3 cache without cached rows has no range B: the bf16 kernel runs
+  const bool use_f8 = h->f8 && h->rows_pad > 0;
+  if (use_f8) {
+    void* sc = nullptr;
+    refcache_fp8_ptr(h, layer, const_cast<void**>(&f8.k8), const_cast<void**>(&f8.vt8), &sc, &f8.rows_pad);
+    f8.scales = static_cast<const float4*>(sc);
+  } else if (!h->f8) {
+    refcache_kv_ptr(h, layer, &kslot, &vslot, nullptr);
+  }
   Operands op{q_live, h->live_rows, k_live, v_live, h->live_rows, kslot, vslot, h->cache_rows, o_live, lse_live};
   return run_attention(h->d_step, h->n_step, h->H, h->D, op, softmax_scale, info, static_cast<cudaStream_t>(stream),
-                       h->step_items.items ? &h->step_items : nullptr);
+                       h->step_items.items ? &h->step_items : nullptr, use_f8 ? &f8 : nullptr);
 }
 
 int full_attention(int batch, int num_heads, int head_dim, const int32_t* cu_seqlens, const void* q, const void* k,

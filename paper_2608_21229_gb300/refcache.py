@@ -24,12 +24,13 @@ ERR_TIMEOUT = -6
 
 MASK_MODES = {"beyond": 0, "beyond_alt": 1, "isolated": 2}
 KERNELS = {"tcgen05": 0, "mma_sync": 1}
+CACHE_DTYPES = {"bf16": 0, "fp8": 0x100}  # REFCACHE_CACHE_FP8: E4M3 codes with per-tile scales
 
 EXPORTED = (
     "refcache_bytes", "refcache_create", "refcache_destroy", "refcache_kv_ptr", "refcache_layer_built",
     "refcache_build", "step_attention", "full_attention", "refcache_status", "refcache_set_wait_timeout_ns",
     "refcache_set_kernel", "refcache_debug_skip_first_load", "refcache_last_error", "refcache_version",
-    "full_attention_noalloc", "refcache_call_launches",
+    "full_attention_noalloc", "refcache_call_launches", "refcache_fp8_ptr",
 )
 NOALLOC_MAX_TASKS = 16384
 
@@ -73,6 +74,8 @@ def load(path: Optional[str] = None):
     L.refcache_destroy.argtypes = [vp]
     L.refcache_destroy.restype = None
     L.refcache_kv_ptr.argtypes = [vp, i32, ctypes.POINTER(vp), ctypes.POINTER(vp), ctypes.POINTER(i64)]
+    L.refcache_fp8_ptr.argtypes = [vp, i32, ctypes.POINTER(vp), ctypes.POINTER(vp), ctypes.POINTER(vp),
+                                   ctypes.POINTER(i64)]
     L.refcache_layer_built.argtypes = [vp, i32]
     L.refcache_call_launches.argtypes = [vp, i32]
     L.refcache_build.argtypes = [vp, i32, vp, vp, vp, vp, vp, f32, vp]
@@ -197,23 +200,26 @@ class RefCache:
     handed to refcache_create, so the library itself allocates nothing.
     """
 
-    def __init__(self, seg: Segments, num_layers: int = 1, mask_mode: str = "beyond", device=None):
+    def __init__(self, seg: Segments, num_layers: int = 1, mask_mode: str = "beyond", device=None,
+                 cache_dtype: str = "bf16"):
         import torch
 
         L = load()
         self.seg, self.num_layers, self.mask_mode = seg, int(num_layers), mask_mode
-        nbytes = L.refcache_bytes(self.num_layers, MASK_MODES[mask_mode], ctypes.byref(seg.c))
+        self.cache_dtype = cache_dtype
+        flags = MASK_MODES[mask_mode] | CACHE_DTYPES[cache_dtype]
+        nbytes = L.refcache_bytes(self.num_layers, flags, ctypes.byref(seg.c))
         if nbytes == 0:
             # the planner rejected the arguments: surface its message
             h = ctypes.c_void_p()
-            _check(L.refcache_create(ctypes.byref(h), self.num_layers, MASK_MODES[mask_mode],
-                                     ctypes.byref(seg.c), ctypes.c_void_p(1), 0))
+            _check(L.refcache_create(ctypes.byref(h), self.num_layers, flags, ctypes.byref(seg.c),
+                                     ctypes.c_void_p(1), 0))
         device = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
         self.mem = torch.empty(nbytes, dtype=torch.uint8, device=device)
         self.h = ctypes.c_void_p()
         with torch.cuda.device(device):
-            _check(L.refcache_create(ctypes.byref(self.h), self.num_layers, MASK_MODES[mask_mode],
-                                     ctypes.byref(seg.c), ctypes.c_void_p(self.mem.data_ptr()), nbytes))
+            _check(L.refcache_create(ctypes.byref(self.h), self.num_layers, flags, ctypes.byref(seg.c),
+                                     ctypes.c_void_p(self.mem.data_ptr()), nbytes))
 
     def close(self):
         if getattr(self, "h", None) is not None and self.h.value:
@@ -241,6 +247,25 @@ class RefCache:
             return self.mem[off:off + n].view(torch.bfloat16).view(rows.value, H, D)
 
         return view(k), view(v)
+
+    def fp8(self, layer: int):
+        """E4M3 cache of a layer as views of the cache memory: (K codes uint8
+        [rows_pad, H, D], V codes uint8 [H, D, rows_pad], scales float32
+        [rows_pad / 128, H, 4] = (s_K, s_V, log2 s_V, 1 / s_V))."""
+        import torch
+
+        k, v, sc, rows = ctypes.c_void_p(), ctypes.c_void_p(), ctypes.c_void_p(), ctypes.c_int64()
+        _check(load().refcache_fp8_ptr(self.h, layer, ctypes.byref(k), ctypes.byref(v), ctypes.byref(sc),
+                                       ctypes.byref(rows)))
+        H, D, n = self.seg.num_heads, self.seg.head_dim, rows.value
+        base = self.mem.data_ptr()
+
+        def view(p, nbytes):
+            off = p.value - base
+            return self.mem[off:off + nbytes]
+
+        return (view(k, n * H * D).view(n, H, D), view(v, n * H * D).view(H, D, n),
+                view(sc, (n // 128) * H * 16).view(torch.float32).view(n // 128, H, 4))
 
     def built(self, layer: int) -> bool:
         r = load().refcache_layer_built(self.h, layer)

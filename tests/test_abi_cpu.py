@@ -120,3 +120,29 @@ def test_binding_fails_loudly_without_library(tmp_path):
             rcb.load(str(tmp_path / "missing.so"))
         finally:
             rcb._lib = saved
+
+
+@pytest.mark.parametrize("w", [workloads.EDIT_1024_5REF, workloads.RAGGED_4REQ, workloads.CFG_SMALL],
+                         ids=lambda w: w.name)
+@pytest.mark.parametrize("mode", ["beyond", "beyond_alt"])
+def test_fp8_cache_bytes_follow_the_padded_layout(lib, w, mode):
+    """E4M3 cache: per layer the K codes and the transposed V codes of every
+    request's cached rows padded to 128, and (s_K, s_V) per tile and head."""
+    s = seg_of(w)
+    layers = 2
+    flags = rcb.MASK_MODES[mode] | rcb.CACHE_DTYPES["fp8"]
+    n = lib.refcache_bytes(layers, flags, ctypes.byref(s.c))
+    rows_pad = sum((r.n_r + (r.n_st if mode == "beyond_alt" else 0) + 127) // 128 * 128 for r in w.requests)
+    align = lambda x: (x + 255) // 256 * 256  # noqa: E731
+    per_layer = 2 * align(rows_pad * w.num_heads * w.head_dim) + align(rows_pad // 128 * w.num_heads * 16)
+    assert layers * per_layer <= n <= layers * per_layer + 64 * 1024
+    bf16 = lib.refcache_bytes(layers, rcb.MASK_MODES[mode], ctypes.byref(s.c))
+    assert n < 0.6 * bf16  # about half the bytes of the bf16 cache
+
+
+def test_fp8_cache_needs_head_dim_128(lib):
+    s = seg_of(workloads.TINY)  # head_dim 64
+    assert lib.refcache_bytes(1, rcb.CACHE_DTYPES["fp8"], ctypes.byref(s.c)) == 0
+    h = ctypes.c_void_p()
+    assert lib.refcache_create(ctypes.byref(h), 1, rcb.CACHE_DTYPES["fp8"], ctypes.byref(s.c), None, 0) == \
+        rcb.ERR_UNSUPPORTED
