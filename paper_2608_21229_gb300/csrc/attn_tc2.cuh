@@ -85,19 +85,27 @@ namespace rc {
 namespace tc2 {
 using tc::Ctl;
 constexpr int kD = 128;
-constexpr int kThreads = 224;
 constexpr int kStages = 4;                  // ring stages (pair_done has as many barriers)
 constexpr uint32_t kKHalf = 64 * 128 * 2;   // 16 KB: this CTA's 64 keys x 128 d of a K tile
 constexpr uint32_t kVHalf = 128 * 64 * 2;   // 16 KB: 128 keys x this CTA's 64 d of a V tile
 constexpr uint32_t kStage = kKHalf + kVHalf;
 constexpr uint32_t kQTile = 128 * 128 * 2;
 constexpr uint32_t kKBox = 64 * 128;        // one K box: 64 rows x 128 bytes
-constexpr int kWarpArrivals = 8;            // 4 softmax warps in each of the 2 CTAs
-constexpr int kProducerWarp = 4, kMmaWarp = 5, kGateWarp = 6;
+// Warp roles: softmax warps first (4, or 8 in the E4M3 kernel, two per SM
+// sub-partition), then the producer, the MMA warp and the gate warp.
+template <bool kF8>
+struct Cfg {
+  static constexpr int kHalves = kF8 ? 2 : 1;         // softmax warps per 32 rows
+  static constexpr int kSoftmaxWarps = 4 * kHalves;
+  static constexpr int kProducerWarp = kSoftmaxWarps, kMmaWarp = kSoftmaxWarps + 1, kGateWarp = kSoftmaxWarps + 2;
+  static constexpr int kThreads = 32 * (kSoftmaxWarps + 3);
+  static constexpr int kWarpArrivals = 2 * kSoftmaxWarps;  // p_full / q8_full: every softmax warp of both CTAs
+};
 constexpr uint32_t kGateBarrier = 1;  // named barrier of the MMA and gate warps (0 is __syncthreads)
 constexpr uint32_t kKHalf8 = 64 * 128;   // 8 KB: this CTA's 64 keys x 128 d of an E4M3 K tile
 constexpr uint32_t kVHalf8 = 64 * 128;   // 8 KB: this CTA's 64 d x 128 keys of an E4M3 V^T tile
 constexpr uint32_t kQ8Tile = 128 * 128;  // this CTA's 128 query rows as E4M3
+constexpr int kScaleSlots = 8;           // ring of per-tile scales of cached tiles (E4M3 kernel)
 static_assert(kStages == 4, "pair_done indexing assumes four stages");
 
 template <bool kF8>
@@ -105,10 +113,13 @@ struct SmemT {
   static constexpr uint32_t kQ = 0;                // Q buffers 0 and 1 (this CTA's 128 rows)
   static constexpr uint32_t kRing = 2 * kQTile;    // stage s: [K half | V half]
   static constexpr uint32_t kQ8 = kRing + kStages * kStage;  // E4M3 Q tile (kF8 only)
-  static constexpr uint32_t kScales = kQ8 + (kF8 ? kQ8Tile : 0u);  // per softmax warp: 2 x 16 B (kF8 only)
-  static constexpr uint32_t kBars = kScales + (kF8 ? 4u * 32u : 0u);
+  static constexpr uint32_t kScales = kQ8 + (kF8 ? kQ8Tile : 0u);  // ring of kScaleSlots x 16 B (kF8 only)
+  static constexpr uint32_t kLX = kScales + (kF8 ? kScaleSlots * 16u : 0u);  // [2][128] fp32 partial row sums
+  static constexpr uint32_t kBars = kLX + (kF8 ? 2u * 128u * 4u : 0u);
   static constexpr int kQFull = 0, kQEmpty = 2, kStageFull = 4, kPairDone = 4 + kStages, kPFull = kPairDone + 4,
-                       kMmaDone = kPFull + 2, kQ8Full = kMmaDone + 1, kNumBars = kQ8Full + 1;
+                       kMmaDone = kPFull + 2, kQ8Full = kMmaDone + 1, kLXFull = kQ8Full + 1,
+                       kScaleFull = kLXFull + 1, kScaleEmpty = kScaleFull + kScaleSlots,
+                       kNumBars = kScaleEmpty + kScaleSlots;
   static constexpr uint32_t kTmemHolder = kBars + 8 * kNumBars;
   static constexpr uint32_t kAbort = kTmemHolder + 4;
   static constexpr uint32_t kUsed = kAbort + 4;
@@ -143,7 +154,7 @@ __device__ __forceinline__ bool wait_cl_warp(uint32_t bar, uint32_t parity, cons
 }  // namespace tc2
 
 template <bool kF8>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThreads, 1)
     attn_tc2_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_ka,
                     const __grid_constant__ CUtensorMap tm_va, const __grid_constant__ CUtensorMap tm_kb,
                     const __grid_constant__ CUtensorMap tm_vb, const AttnArgs args) {
@@ -154,7 +165,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
   using tc2::kStage;
   using tc2::kStages;
   using tc2::kVHalf;
-  using tc2::kWarpArrivals;
+  using Cfg = tc2::Cfg<kF8>;
+  constexpr int kWarpArrivals = Cfg::kWarpArrivals;
   using tc2::group_parity;
   using tc2::wait_cl;
   using tc2::wait_cl_warp;
@@ -198,11 +210,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
     }
     mbar_init(bar(L::kMmaDone), 1);
     mbar_init(bar(L::kQ8Full), kWarpArrivals);
+    mbar_init(bar(L::kLXFull), Cfg::kSoftmaxWarps);
+    for (int s = 0; s < tc2::kScaleSlots; ++s) {
+      mbar_init(bar(L::kScaleFull + s), 1);
+      mbar_init(bar(L::kScaleEmpty + s), Cfg::kSoftmaxWarps);
+    }
     *abort_flag = 0;
     fence_barrier_init();
     fence_proxy_async_smem();
   }
-  if (warp == tc2::kMmaWarp) {
+  if (warp == Cfg::kMmaWarp) {
     tmem_alloc_pair(smem_u32(tmem_holder), kTmemCols);
     tmem_relinquish_pair();
   }
@@ -214,7 +231,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
   const Ctl ctl{abort_flag, args.timeout_ns};
   auto lbar = [&](int i) -> uint32_t { return mapa_shared(bar(i), 0); };  // leader's barrier i
 
-  if (warp == tc2::kProducerWarp) {
+  if (warp == Cfg::kProducerWarp) {
     // ------------------------------------------------------------ producer (both CTAs)
     // This CTA's halves of the stages of every group, in group order, and an
     // item's Q rows just before its first stage.
@@ -222,8 +239,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
       int armed_phase[kStages];
       for (int s = 0; s < kStages; ++s) armed_phase[s] = -1;
       int q_armed[2] = {-1, -1};
+      int scale_armed[tc2::kScaleSlots];
+      for (int s = 0; s < tc2::kScaleSlots; ++s) scale_armed[s] = -1;
       bool skip_next = leader && args.dbg_skip_first_load != 0;
-      int g = 0, qi = 0;
+      int g = 0, qi = 0, si = 0;  // si: cached tiles whose scales went into the ring
       Task tk;
       int head = 0, na = 0;
       // stage of group g: K tile kj (if kj >= 0) and V tile vj (if vj >= 0) of the item
@@ -238,6 +257,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         const bool k8 = kF8 && kj >= 0 && ks.in_b, v8 = kF8 && vj >= 0 && vs.in_b;
         const uint32_t bytes =
             2 * ((kj >= 0 ? (k8 ? kKHalf8 : kKHalf) : 0u) + (vj >= 0 ? (v8 ? kVHalf8 : kVHalf) : 0u));
+        if (k8) {
+          // this CTA's softmax warps read the cached tile's scales from ring slot
+          // si % kScaleSlots; the slot's previous tile must have been read
+          const int sl = si % tc2::kScaleSlots, use = si / tc2::kScaleSlots;
+          if (use > 0 && !wait_one(bar(L::kScaleEmpty + sl), static_cast<uint32_t>(use - 1) & 1u, ctl, 16)) return false;
+          mbar_arrive_expect_tx(bar(L::kScaleFull + sl), 16u);
+          scale_armed[sl] = use & 1;
+          bulk_load(base + L::kScales + 16u * static_cast<uint32_t>(sl),
+                    args.b_scales + ((tk.b_row0 >> 7) + (kj - na)) * args.num_heads + head, 16u,
+                    bar(L::kScaleFull + sl));
+          ++si;
+        }
         if (skip_next) {  // fault injection: the leader never arms or loads this stage
           skip_next = false;
         } else {
@@ -293,9 +324,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
           drain_one(bar(L::kStageFull + s), static_cast<uint32_t>(armed_phase[s]), args.timeout_ns);
       for (int b = 0; b < 2; ++b)
         if (q_armed[b] >= 0) drain_one(bar(L::kQFull + b), static_cast<uint32_t>(q_armed[b]) & 1u, args.timeout_ns);
+      for (int s = 0; s < tc2::kScaleSlots; ++s)
+        if (scale_armed[s] >= 0) drain_one(bar(L::kScaleFull + s), static_cast<uint32_t>(scale_armed[s]), args.timeout_ns);
     }
     __syncwarp();
-  } else if (warp == tc2::kMmaWarp) {
+  } else if (warp == Cfg::kMmaWarp) {
     // ------------------------------------------------------------ MMA warp (leader)
     if (leader) {
       // descriptors of stage 0 (stage s: + s * kStage / 16) and of Q buffer 0
@@ -410,7 +443,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
       }
     }
     __syncwarp();
-  } else if (warp == tc2::kGateWarp) {
+  } else if (warp == Cfg::kGateWarp) {
     // ------------------------------------------------------------ gate warp (leader)
     // The same group sequence as the MMA warp; every wait is bounded, and a
     // failed wait is passed on through the handshake, after which both leave.
@@ -445,13 +478,27 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------ softmax (both CTAs)
-    const int trow = warp * 32 + lane;                     // row within this CTA's 128 rows (= TMEM lane)
+    // kH = 1: warp w (0-3) owns rows 32 w .. 32 w + 31 of this CTA's 128 rows
+    // (its TMEM lanes) and all 128 key columns.  kH = 2 (E4M3 kernel): warps w
+    // and w + 4 share those rows, warp w + 4 hh taking key columns and O
+    // columns [64 hh, 64 hh + 64), so that two warps per SM sub-partition share
+    // the exponentials.  Both read the whole S row, find the same row maximum
+    // and take the same rescale decisions; their partial row sums meet in the
+    // epilogue through shared memory.
+    constexpr int kH = Cfg::kHalves;
+    constexpr int kC = 128 / kH;  // key columns and O columns of this thread
+    const int quarter = warp & 3, hh = warp >> 2;
+    const int col0 = hh * kC;
+    const int trow = quarter * 32 + lane;                  // row within this CTA's 128 rows (= TMEM lane)
     const int prow = 128 * static_cast<int>(rank) + trow;  // row within the item
-    const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
+    const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
     const float sl2 = args.scale_log2;
     const f32x2 sl2x2 = make_f32x2(sl2, sl2);
-    int t = 0;  // tiles of earlier items
-    int G = 0;  // first group of the item
+    float* lx = reinterpret_cast<float*>(base_ptr + L::kLX);  // [2][128] partial row sums (kH = 2)
+    int t = 0;     // tiles of earlier items
+    int G = 0;     // first group of the item
+    int n_lx = 0;  // row-sum exchanges so far (kH = 2)
+    int si = 0;    // cached tiles read from the scale ring so far
     // wait until group g is complete (both CTAs see the multicast commit)
     auto wait_group = [&](int g, int where) -> bool {
       return wait_cl_warp(bar(L::kPairDone + (g & 3)), group_parity(g), ctl, where);
@@ -464,12 +511,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
       const int nkv = n_key_tiles(tk, na);
       const bool row_ok = prow < tk.q_rows;
       const int64_t grow = static_cast<int64_t>(tk.q_row0) + prow;
-      __nv_bfloat16* orow = args.out + grow * args.row_stride + static_cast<int64_t>(head) * D;
+      __nv_bfloat16* orow = args.out + grow * args.row_stride + static_cast<int64_t>(head) * D + col0;
       if (nkv == 0) {
         if (row_ok) {
           uint4 z = make_uint4(0, 0, 0, 0);
-          for (int c = 0; c < D / 8; ++c) reinterpret_cast<uint4*>(orow)[c] = z;
-          if (args.lse) args.lse[grow * args.num_heads + head] = -INFINITY;
+          for (int c = 0; c < kC / 8; ++c) reinterpret_cast<uint4*>(orow)[c] = z;
+          if (args.lse && hh == 0) args.lse[grow * args.num_heads + head] = -INFINITY;
         }
         continue;
       }
@@ -480,6 +527,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
       if (kF8 && nkv > na) {
         // quantise this thread's query row of this head into the E4M3 Q tile:
         // s = amax / 448, code = E4M3(x * (448 / amax)), round to nearest even
+        // (the maximum over the whole row; each half writes its own columns)
         uint4 raw[16];
         if (row_ok) {
           const uint4* src = reinterpret_cast<const uint4*>(args.q + grow * args.row_stride + static_cast<int64_t>(head) * D);
@@ -501,6 +549,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         const uint32_t q8_row = base + L::kQ8 + static_cast<uint32_t>(trow) * 128u;
 #pragma unroll
         for (int c = 0; c < 8; ++c) {  // 16 codes per 16-byte chunk, 128-byte swizzle
+          if (kH == 2 && (c >> 2) != hh) continue;
           uint32_t w[4];
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
@@ -521,14 +570,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         s_ref = sc0.y > 0.f ? sc0.y : 1.f;
         l2_ref = sc0.y > 0.f ? sc0.z : 0.f;
       }
-      // the scales of cached tiles are fetched one tile ahead by asynchronous
-      // copies into this warp's two slots (an ordinary load still in flight
-      // would hold up the release of the next P arrival)
-      const uint32_t sc_slots = base + L::kScales + static_cast<uint32_t>(warp) * 32u;
-      if (kF8 && na < nkv) {
-        if (lane == 0) cp_async_16(sc_slots, args.b_scales + scale_row0);
-        cp_async_commit();
-      }
       for (int j = 0; j < nkv; ++j, ++t) {
         const int b = t & 1;
         const TileSrc src = tile_src(tk, na, j);
@@ -537,18 +578,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         const bool t8 = kF8 && j >= na;
         float c_t = sl2, shift = 0.f, wshift = -l2_ref, lscale = s_ref;
         if (t8) {
-          const int jb = j - na;  // index among the item's cached tiles
-          if (j + 1 < nkv) {
-            if (lane == 0)
-              cp_async_16(sc_slots + 16u * static_cast<uint32_t>((jb + 1) & 1),
-                          args.b_scales + scale_row0 + (jb + 1) * args.num_heads);
-            cp_async_commit();
-            cp_async_wait<1>();
-          } else {
-            cp_async_wait<0>();
-          }
+          // the producer's ring of tile scales (no global access here: an
+          // ordinary load still in flight would hold up the next P arrival)
+          const int sl = si % tc2::kScaleSlots;
+          if (!wait_warp(bar(L::kScaleFull + sl), static_cast<uint32_t>(si / tc2::kScaleSlots) & 1u, ctl, 17))
+            goto softmax_done;
+          const float4 sc = ld_shared_f4(base + L::kScales + 16u * static_cast<uint32_t>(sl));
           __syncwarp();
-          const float4 sc = ld_shared_f4(sc_slots + 16u * static_cast<uint32_t>(jb & 1));
+          if (lane == 0) mbar_arrive(bar(L::kScaleEmpty + sl));
+          ++si;
           c_t = fmaxf(c_row * sc.x, 1e-30f);
           // delta = log2(s_V / s_ref); an all-zero V tile (s_V = 0) takes delta = 0
           const bool nz = sc.y > 0.f;
@@ -560,8 +598,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         if (!wait_group(G + j, 8)) goto softmax_done;
         tc_fence_after();
         const uint32_t t_s = tmem + lane_off + kColS + 128u * b;
-        float s[128];
-        {
+        // this thread's columns of S in s[], the row maximum of the raw scores in m_raw
+        float s[kC];
+        float m_raw;
+        if constexpr (kH == 1) {
           uint32_t r0[32], r1[32], r2[32], r3[32];
           tmem_ld32(t_s + 0u, r0);
           tmem_ld32(t_s + 32u, r1);
@@ -578,22 +618,64 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
             s[64 + c] = __uint_as_float(r2[c]);
             s[96 + c] = __uint_as_float(r3[c]);
           }
-        }
-        if (src.valid < 128) {  // keys past the end of the range
+          if (src.valid < 128) {  // keys past the end of the range
 #pragma unroll
-          for (int c = 0; c < 128; ++c)
-            if (c >= src.valid) s[c] = -INFINITY;
-        }
-        // row maximum: four independent chains of 3-input max
-        float mx[4];
+            for (int c = 0; c < 128; ++c)
+              if (c >= src.valid) s[c] = -INFINITY;
+          }
+          // four independent chains of 3-input max
+          float mx[4];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          mx[k] = fmax3(s[32 * k], s[32 * k + 1], s[32 * k + 2]);
+          for (int k = 0; k < 4; ++k) {
+            mx[k] = fmax3(s[32 * k], s[32 * k + 1], s[32 * k + 2]);
 #pragma unroll
-          for (int c = 3; c < 31; c += 2) mx[k] = fmax3(mx[k], s[32 * k + c], s[32 * k + c + 1]);
-          mx[k] = fmaxf(mx[k], s[32 * k + 31]);
+            for (int c = 3; c < 31; c += 2) mx[k] = fmax3(mx[k], s[32 * k + c], s[32 * k + c + 1]);
+            mx[k] = fmaxf(mx[k], s[32 * k + 31]);
+          }
+          m_raw = fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
+        } else {
+          // own 64 columns, and the other half's 64 for the maximum only
+          const uint32_t other = static_cast<uint32_t>(kC - col0);
+          uint32_t r0[32], r1[32], x0[32], x1[32];
+          tmem_ld32(t_s + static_cast<uint32_t>(col0), r0);
+          tmem_ld32(t_s + static_cast<uint32_t>(col0) + 32u, r1);
+          tmem_ld32(t_s + other, x0);
+          tmem_ld32(t_s + other + 32u, x1);
+          tmem_wait_ld(r0);
+          tmem_wait_ld(r1);
+          tmem_wait_ld(x0);
+          tmem_wait_ld(x1);
+          float o[64];
+#pragma unroll
+          for (int c = 0; c < 32; ++c) {
+            s[c] = __uint_as_float(r0[c]);
+            s[32 + c] = __uint_as_float(r1[c]);
+            o[c] = __uint_as_float(x0[c]);
+            o[32 + c] = __uint_as_float(x1[c]);
+          }
+          if (src.valid < 128) {  // keys past the end of the range
+#pragma unroll
+            for (int c = 0; c < 64; ++c) {
+              if (col0 + c >= src.valid) s[c] = -INFINITY;
+              if (static_cast<int>(other) + c >= src.valid) o[c] = -INFINITY;
+            }
+          }
+          float mx[4];
+#pragma unroll
+          for (int k = 0; k < 2; ++k) {
+            mx[k] = fmax3(s[32 * k], s[32 * k + 1], s[32 * k + 2]);
+            mx[2 + k] = fmax3(o[32 * k], o[32 * k + 1], o[32 * k + 2]);
+#pragma unroll
+            for (int c = 3; c < 31; c += 2) {
+              mx[k] = fmax3(mx[k], s[32 * k + c], s[32 * k + c + 1]);
+              mx[2 + k] = fmax3(mx[2 + k], o[32 * k + c], o[32 * k + c + 1]);
+            }
+            mx[k] = fmaxf(mx[k], s[32 * k + 31]);
+            mx[2 + k] = fmaxf(mx[2 + k], o[32 * k + 31]);
+          }
+          m_raw = fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
         }
-        const float m_tile = fmaf(fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3])), c_t, shift);
+        const float m_tile = fmaf(m_raw, c_t, shift);
         if (j == 0) {
           m_run = m_tile;
         } else if (__any_sync(0xffffffffu, m_tile > m_run + 8.0f)) {
@@ -605,9 +687,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
           const f32x2 alpha2 = make_f32x2(alpha, alpha);
           m_run = m_new;
           l_run *= alpha;
-          const uint32_t t_o = tmem + lane_off + kColO;
+          const uint32_t t_o = tmem + lane_off + kColO + static_cast<uint32_t>(col0);
 #pragma unroll
-          for (int cc = 0; cc < D / 16; ++cc) {
+          for (int cc = 0; cc < kC / 16; ++cc) {
             uint32_t o[16];
             tmem_ld16(t_o + 16u * cc, o);
             tmem_wait_ld(o);
@@ -633,7 +715,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         for (int i = 0; i < 4; ++i) lacc[i] = make_f32x2(0.f, 0.f);
         if (t8) {
 #pragma unroll
-          for (int k = 0; k < 4; ++k) {
+          for (int k = 0; k < kC / 32; ++k) {
             uint32_t pk[8];
 #pragma unroll
             for (int c = 0; c < 8; ++c) {
@@ -647,11 +729,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
               lacc[(2 * c + 1) & 3] = add_f32x2(lacc[(2 * c + 1) & 3], make_f32x2(x2, x3));
               pk[c] = pack_e4m3x4(x0, x1, x2, x3);
             }
-            tmem_st8(t_p + 8u * k, pk);
+            tmem_st8(t_p + static_cast<uint32_t>(col0 / 4) + 8u * k, pk);
           }
         } else {
 #pragma unroll
-          for (int k = 0; k < 4; ++k) {
+          for (int k = 0; k < kC / 32; ++k) {
             uint32_t pk[16];
 #pragma unroll
             for (int c = 0; c < 16; ++c) {
@@ -662,7 +744,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
               lacc[c & 3] = add_f32x2(lacc[c & 3], make_f32x2(x, y));
               pk[c] = pack_bf16x2(x, y);
             }
-            tmem_st16(t_p + 16u * k, pk);
+            tmem_st16(t_p + static_cast<uint32_t>(col0 / 2) + 16u * k, pk);
           }
         }
         {
@@ -684,14 +766,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
       {
         if (!wait_group(G + nkv + 1, 10)) goto softmax_done;  // the item's last group
         tc_fence_after();
-        const float inv_l = kF8 ? s_ref / l_run : 1.0f / l_run;
-        const uint32_t t_o = tmem + lane_off + kColO;
+        float l_tot = l_run;
+        if constexpr (kH == 2) {
+          // the two halves' partial row sums (relative to the same maximum)
+          lx[hh * 128 + trow] = l_run;
+          __syncwarp();
+          if (lane == 0) mbar_arrive(bar(L::kLXFull));
+          if (!wait_warp(bar(L::kLXFull), static_cast<uint32_t>(n_lx) & 1u, ctl, 15)) goto softmax_done;
+          ++n_lx;
+          l_tot = l_run + lx[(1 - hh) * 128 + trow];
+        }
+        const float inv_l = kF8 ? s_ref / l_tot : 1.0f / l_tot;
+        const uint32_t t_o = tmem + lane_off + kColO + static_cast<uint32_t>(col0);
         if (tk.part > 0) {
           // a part of a split item: O / l in fp32 and m + log l to its workspace slot
           const int64_t prow_ws = static_cast<int64_t>(tk.part - 1) * args.rows_per_task + prow;
-          float4* dst = reinterpret_cast<float4*>(args.part_o + prow_ws * D);
+          float4* dst = reinterpret_cast<float4*>(args.part_o + prow_ws * D + col0);
 #pragma unroll
-          for (int cc = 0; cc < D / 32; ++cc) {
+          for (int cc = 0; cc < kC / 32; ++cc) {
             uint32_t o[32];
             tmem_ld32(t_o + 32u * cc, o);
             tmem_wait_ld(o);
@@ -704,13 +796,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
             }
           }
           tc_fence_before();
-          if (row_ok) args.part_lse[prow_ws] = (m_run + log2f(l_run)) * 0.69314718055994530942f;
+          if (row_ok && hh == 0) args.part_lse[prow_ws] = (m_run + log2f(l_tot)) * 0.69314718055994530942f;
           G += nkv + 2;
           continue;
         }
-        uint32_t packed[D / 2];
+        uint32_t packed[kC / 2];
 #pragma unroll
-        for (int cc = 0; cc < D / 32; ++cc) {
+        for (int cc = 0; cc < kC / 32; ++cc) {
           uint32_t o[32];
           tmem_ld32(t_o + 32u * cc, o);
           tmem_wait_ld(o);
@@ -725,9 +817,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
         if (row_ok) {
           uint4* dst = reinterpret_cast<uint4*>(orow);
 #pragma unroll
-          for (int c = 0; c < D / 8; ++c)
+          for (int c = 0; c < kC / 8; ++c)
             dst[c] = make_uint4(packed[4 * c], packed[4 * c + 1], packed[4 * c + 2], packed[4 * c + 3]);
-          if (args.lse) args.lse[grow * args.num_heads + head] = (m_run + log2f(l_run)) * 0.69314718055994530942f;
+          if (args.lse && hh == 0)
+            args.lse[grow * args.num_heads + head] = (m_run + log2f(l_tot)) * 0.69314718055994530942f;
         }
       }
       G += nkv + 2;
@@ -738,7 +831,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::kThreads, 1)
   tc_fence_before();
   __syncthreads();
   cluster_sync();  // the pair's MMAs and TMEM reads are over in both CTAs
-  if (warp == tc2::kMmaWarp) {
+  if (warp == Cfg::kMmaWarp) {
     tc_fence_after();
     tmem_dealloc_pair(tmem, kTmemCols);
   }

@@ -223,7 +223,7 @@ int tc2_clusters(DeviceInfo* info, int* clusters_out) {
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_tc2_kernel)");
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3(2 * static_cast<unsigned>(info->num_sms / 2), 1, 1);
-    cfg.blockDim = dim3(rc::tc2::kThreads, 1, 1);
+    cfg.blockDim = dim3(rc::tc2::Cfg<kF8>::kThreads, 1, 1);
     cfg.dynamicSmemBytes = smem;
     int clusters = 0;
     e = cudaOccupancyMaxActiveClusters(&clusters, rc::attn_tc2_kernel<kF8>, &cfg);
@@ -244,7 +244,7 @@ int launch_tc2(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info
   if (rc) return rc;
   const int clusters = std::min(a.n_items, max_clusters);
   rc::attn_tc2_kernel<kF8>
-      <<<2 * clusters, rc::tc2::kThreads, smem, s>>>(maps[0], maps[1], maps[2], maps[3], maps[4], a);
+      <<<2 * clusters, rc::tc2::Cfg<kF8>::kThreads, smem, s>>>(maps[0], maps[1], maps[2], maps[3], maps[4], a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "attn_tc2_kernel launch");
   return REFCACHE_OK;
