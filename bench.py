@@ -205,7 +205,7 @@ def run_ours(args, ws, rank, local):
     w = workloads.ALL[args.workload]
     H, D = w.num_heads, w.head_dim
     seg = rcb.Segments.from_workload(w)
-    cache = rcb.RefCache(seg, num_layers=1, mask_mode="beyond", device=dev)
+    cache = rcb.RefCache(seg, num_layers=1, mask_mode="beyond", device=dev, cache_dtype=args.cache)
     scale = 1.0 / math.sqrt(D)
     qs, ks, vs = (t.to(dev) for t in workloads.static_qkv(w))
     lives = [tuple(t.to(dev) for t in workloads.live_qkv(w, step=i)) for i in range(N_LIVE_SETS)]
@@ -269,6 +269,9 @@ def run_ours(args, ws, rank, local):
     cfg = None
     if w.name == "edit1024_5ref" and not args.no_cfg:
         cfg = time_cfg_pair(dev, stream, scale, t_step)
+    fp8 = None
+    if w.name == "edit1024_5ref" and not args.no_fp8 and args.cache == "bf16":
+        fp8 = time_fp8_cache(w, dev, stream, scale, t_step)
     linear = None
     if not args.no_linear and t_full == t_full:
         linear = linear_accounting(w, dev, stream, t_pre, t_step, t_full)
@@ -279,6 +282,9 @@ def run_ours(args, ws, rank, local):
     flops_all, secs_all = aggregate(flops_per_step * args.steps, total_s, ws)
     pk = peaks()
     achieved = step_flops / t_step / 1e12
+    # the E4M3 cache's cached tiles run on E4M3 MMAs: their peak is the bf16
+    # measurement times the nominal E4M3 / bf16 ratio (2)
+    peak_mult = 2.0 if args.cache == "fp8" else 1.0
     line = {
         "metric": METRIC,
         "value": flops_all / secs_all / 1e12,
@@ -290,9 +296,9 @@ def run_ours(args, ws, rank, local):
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
-        "dtype": "bf16",
+        "dtype": "bf16" if args.cache == "bf16" else "e4m3 cache, bf16 live",
         "data": "synthetic",
-        "config": workload_config(w, args.kernel, ws),
+        "config": dict(workload_config(w, args.kernel, ws), cache=args.cache),
         "step_attention": {"ms": t_step * 1e3, "tflops": achieved, "flops": step_flops},
         "prefill": {"ms": t_pre * 1e3, "tflops": pre_flops / t_pre / 1e12, "flops": pre_flops},
         "full_attention": {"ms": t_full * 1e3, "tflops": full_flops / t_full / 1e12, "flops": full_flops}
@@ -306,16 +312,20 @@ def run_ours(args, ws, rank, local):
             "kernel": ("attn_mma_kernel (mma.sync)" if args.kernel == "mma_sync" else
                        "attn_tc2_kernel (tcgen05, CTA pairs)" if D == 128 else "attn_tc_kernel<64> (tcgen05)")
                       + " in step_attention",
-            "bound": "tensor", "achieved": achieved, "peak": pk["bf16_sustained"], "unit": "TFLOP/s",
-            "frac": achieved / pk["bf16_sustained"],
-            "peak_kind": f"bf16 dense, {pk['source']} sustained (kernel timed inside a long step)",
-            "frac_of_burst": achieved / pk["bf16_burst"],
-            "traffic": recorded_traffic(w.name, args.kernel),
+            "bound": "tensor", "achieved": achieved, "peak": peak_mult * pk["bf16_sustained"], "unit": "TFLOP/s",
+            "frac": achieved / (peak_mult * pk["bf16_sustained"]),
+            "peak_kind": (f"bf16 dense, {pk['source']} sustained (kernel timed inside a long step)"
+                          if args.cache == "bf16" else
+                          f"E4M3 dense = 2 x bf16 {pk['source']} sustained (nominal ratio)"),
+            "frac_of_burst": achieved / (peak_mult * pk["bf16_burst"]),
+            "traffic": recorded_traffic(w.name, args.kernel) if args.cache == "bf16" else None,
             "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum, one step_attention launch"
                               " (profiles/); null when the kernel sources changed since",
-            "algorithmic_bytes": 2 * (seg.live_rows * H * D * 2) * 2 + acc.cache_bytes(w.requests, H, D),
+            "algorithmic_bytes": 2 * (seg.live_rows * H * D * 2) * 2
+                                 + acc.cache_bytes(w.requests, H, D) // (2 if args.cache == "fp8" else 1),
         },
         "cfg_pair": cfg,
+        "fp8_cache": fp8,
         "linear_accounting": linear,
         "reference_sweep": sweep,
         "ragged_batch": ragged,
@@ -441,6 +451,66 @@ def linear_accounting(w, dev, stream, t_pre, t_step, t_full):
         "cublas_tflops": flops_tok * (S + R) / tl_all / 1e12,
         "modelled_40step_with_linear": full / cached,
         "note": "context only: one layer, attention times measured above, linear work timed with cuBLAS",
+    }
+
+
+def time_fp8_cache(w, dev, stream, scale, t_step_bf16):
+    """The E4M3 reference cache (an approximate variant of the exact cache) on
+    the same workload and inputs as the bf16 step: step time, cache bytes, and
+    the outputs' distance from the exact kernel's on the same inputs."""
+    import torch
+
+    import workloads
+    from paper_2608_21229_gb300 import accounting as acc
+    from paper_2608_21229_gb300 import refcache as rcb
+
+    H, D = w.num_heads, w.head_dim
+    seg = rcb.Segments.from_workload(w)
+    cache = rcb.RefCache(seg, num_layers=1, mask_mode="beyond", device=dev, cache_dtype="fp8")
+    cache16 = rcb.RefCache(seg, num_layers=1, mask_mode="beyond", device=dev)
+    qs, ks, vs = (t.to(dev) for t in workloads.static_qkv(w))
+    lives = [tuple(t.to(dev) for t in workloads.live_qkv(w, step=i)) for i in range(N_LIVE_SETS)]
+    o_s = torch.empty(seg.static_rows, H, D, dtype=torch.bfloat16, device=dev)
+    o_l = torch.empty(seg.live_rows, H, D, dtype=torch.bfloat16, device=dev)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    cache.build(0, qs, ks, vs, o_s, scale=scale)
+    b.record(stream)
+    for i in range(3):
+        cache.step(0, *lives[i % N_LIVE_SETS], o_l, scale=scale)
+    torch.cuda.synchronize()
+    t_build = a.elapsed_time(b) / 1e3
+    n = 2 * T_STEPS
+    a.record(stream)
+    for i in range(n):
+        cache.step(0, *lives[i % N_LIVE_SETS], o_l, scale=scale)
+    b.record(stream)
+    torch.cuda.synchronize()
+    if rcb.status() != rcb.OK:
+        raise RuntimeError(f"device error in the E4M3-cache step: {rcb.last_error()}")
+    t = a.elapsed_time(b) / n / 1e3
+    # distance from the exact (bf16-cache) kernel on live set 0
+    o16 = torch.empty_like(o_l)
+    cache16.build(0, qs, ks, vs, o_s, scale=scale)
+    cache16.step(0, *lives[0], o16, scale=scale)
+    cache.step(0, *lives[0], o_l, scale=scale)
+    torch.cuda.synchronize()
+    d = (o_l.float() - o16.float()).abs()
+    flops = acc.flops(acc.step_units(w.requests), H, D)
+    bf16_bytes = acc.cache_bytes(w.requests, H, D, "beyond")
+    k8, vt8, sc = cache.fp8(0)
+    fp8_bytes = k8.numel() + vt8.numel() + sc.numel() * 4
+    return {
+        "step_ms": t * 1e3,
+        "tflops_equivalent": flops / t / 1e12,
+        "vs_bf16_step": t / t_step_bf16,
+        "build_ms": t_build * 1e3,
+        "cache_mb_per_layer": fp8_bytes / 1e6,
+        "bf16_cache_mb_per_layer": bf16_bytes / 1e6,
+        "max_abs_vs_exact_kernel": float(d.max()),
+        "mean_abs_vs_exact_kernel": float(d.mean()),
+        "note": "approximate variant: cached K/V as E4M3 with per-tile scales, E4M3 tensor-core MMAs for "
+                "cached tiles; same FLOP count as the exact step",
     }
 
 
@@ -681,7 +751,8 @@ def run_reference(args, ws, rank):
     return {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": tot_s / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-            "config": workload_config(w, "cpu oracle (plain fp64 definition) on bounded samples", ws),
+            "config": dict(workload_config(w, "cpu oracle (plain fp64 definition) on bounded samples", ws),
+                           cache=args.cache),
             "cpu_baseline": {"value": v, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -701,6 +772,9 @@ def main(argv=None):
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end measurement")
     ap.add_argument("--no-full", action="store_true", help="skip the full-attention baseline")
     ap.add_argument("--no-cfg", action="store_true", help="skip the guided (positive + negative branch) step")
+    ap.add_argument("--no-fp8", action="store_true", help="skip the E4M3-cache variant")
+    ap.add_argument("--cache", choices=("bf16", "fp8"), default="bf16",
+                    help="format of the main run's reference cache (fp8: the approximate E4M3 variant)")
     ap.add_argument("--no-linear", action="store_true", help="skip the cuBLAS-timed linear-work accounting")
     ap.add_argument("--no-sweep", action="store_true",
                     help="skip the 1024^2 reference sweep (1-10 refs) and the ragged serving batch")
