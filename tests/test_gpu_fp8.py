@@ -195,3 +195,43 @@ def test_fp8_call_launches():
     cache = rcb.RefCache(rcb.Segments.from_workload(w), device="cuda:0", cache_dtype="fp8")
     assert cache.launches("build") >= 2  # quantisation + attention (+ combine)
     assert cache.launches("step") >= 1
+
+
+def test_fp8_layers_are_independent_and_match_single_layer_caches():
+    """A three-layer E4M3 cache: each layer built with its own inputs gives the
+    same cache bytes and step outputs as a one-layer cache of that layer."""
+    w = workloads.CFG_SMALL
+    seg = rcb.Segments.from_workload(w)
+    dev = torch.device("cuda:0")
+    H, D = w.num_heads, w.head_dim
+    multi = rcb.RefCache(seg, num_layers=3, device=dev, cache_dtype="fp8")
+    outs = {}
+    for layer in (2, 0, 1):  # out of order: a layer's build must not touch another's
+        qs, ks, vs = (t.to(dev) for t in workloads.static_qkv(w, layer))
+        o_s = torch.empty_like(qs)
+        multi.build(layer, qs, ks, vs, o_s)
+    for layer in range(3):
+        ql, kl, vl = (t.to(dev) for t in workloads.live_qkv(w, layer))
+        o_l = torch.empty_like(ql)
+        multi.step(layer, ql, kl, vl, o_l)
+        outs[layer] = o_l
+    torch.cuda.synchronize()
+    assert rcb.status() == rcb.OK
+    for layer in range(3):
+        single = rcb.RefCache(seg, num_layers=1, device=dev, cache_dtype="fp8")
+        qs, ks, vs = (t.to(dev) for t in workloads.static_qkv(w, layer))
+        ql, kl, vl = (t.to(dev) for t in workloads.live_qkv(w, layer))
+        o_s, o_l = torch.empty_like(qs), torch.empty_like(ql)
+        single.build(0, qs, ks, vs, o_s)
+        single.step(0, ql, kl, vl, o_l)
+        torch.cuda.synchronize()
+        for a, b in zip(multi.fp8(layer), single.fp8(0)):
+            assert torch.equal(a, b), f"layer {layer}: cache bytes differ"
+        assert torch.equal(outs[layer].view(torch.int16), o_l.view(torch.int16)), f"layer {layer}: outputs differ"
+
+
+def test_fp8_edit1024_10ref_sampled():
+    """The largest reference count of the sweep (40960 cached rows per request)."""
+    w = [x for x in workloads.SWEEP_1024 if x.requests[0].n_r == 10 * 4096][0]
+    run = Fp8Run(w)
+    check_step(run, heads=[3, 22], rows_per_request=24, seed=9)
