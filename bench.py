@@ -723,10 +723,29 @@ def cpu_baseline(w, budget_s=15.0):
     n_step, n_pre = sample_sizes(w, int(64 * scale))
     static, live, sp, pp = oracle_sample(w, n_step, n_pre, seed=1)
     f, s = time_oracle_sample(w, static, live, sp, pp)
-    return {"value": f / s / 1e12, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+    cores = oracle.max_threads()
+    return {"value": f / s / 1e12, "unit": UNIT, "cores": cores, "kind": "oracle",
             "sample": f"{len(sp)} (row, head) outputs of the step and {len(pp)} of the prefill of {w.name}, "
                       f"fp64 plain definition, {s:.1f} s",
-            "seconds": s, "flops": f}
+            "seconds": s, "flops": f, "single_thread": single_thread_oracle(cores)}
+
+
+def single_thread_oracle(cores_after, pairs=512):
+    """The oracle on one host core for the two small workloads (context for
+    the multi-core figure): a bounded sample of each, GFLOP/s."""
+    import oracle
+    import workloads
+
+    out = []
+    oracle.set_threads(1)
+    try:
+        for w in (workloads.TINY, workloads.EDIT_512_2REF):
+            static, live, sp, pp = oracle_sample(w, *sample_sizes(w, pairs), seed=2)
+            f, s = time_oracle_sample(w, static, live, sp, pp)
+            out.append({"workload": w.name, "outputs": int(len(sp) + len(pp)), "seconds": s, "gflops": f / s / 1e9})
+    finally:
+        oracle.set_threads(cores_after)
+    return out
 
 
 def run_reference(args, ws, rank):
