@@ -78,6 +78,9 @@
 // at most 2^8; each tile adds its unshifted weight sum to l, and
 // O = s_ref * acc / l.
 #pragma once
+#ifndef RC_SOFTMAX_MAXFREE
+#define RC_SOFTMAX_MAXFREE 0
+#endif
 #include "attn_tc.cuh"
 
 namespace rc {
@@ -487,6 +490,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
     // epilogue through shared memory.
     constexpr int kH = Cfg::kHalves;
     constexpr int kC = 128 / kH;  // key columns and O columns of this thread
+    // one softmax thread per row: after a row's first tile, exponentials are
+    // taken against the running maximum and checked by their sum
+    constexpr bool kMaxFree = kH == 1 && RC_SOFTMAX_MAXFREE;
     const int quarter = warp & 3, hh = warp >> 2;
     const int col0 = hh * kC;
     const int trow = quarter * 32 + lane;                  // row within this CTA's 128 rows (= TMEM lane)
@@ -598,9 +604,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
         if (!wait_group(G + j, 8)) goto softmax_done;
         tc_fence_after();
         const uint32_t t_s = tmem + lane_off + kColS + 128u * b;
-        // this thread's columns of S in s[], the row maximum of the raw scores in m_raw
+        // this thread's columns of S in s[]; with two halves, the other half's
+        // maximum in m_other
         float s[kC];
-        float m_raw;
+        float m_other = -INFINITY;
         if constexpr (kH == 1) {
           uint32_t r0[32], r1[32], r2[32], r3[32];
           tmem_ld32(t_s + 0u, r0);
@@ -623,16 +630,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
             for (int c = 0; c < 128; ++c)
               if (c >= src.valid) s[c] = -INFINITY;
           }
-          // four independent chains of 3-input max
-          float mx[4];
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            mx[k] = fmax3(s[32 * k], s[32 * k + 1], s[32 * k + 2]);
-#pragma unroll
-            for (int c = 3; c < 31; c += 2) mx[k] = fmax3(mx[k], s[32 * k + c], s[32 * k + c + 1]);
-            mx[k] = fmaxf(mx[k], s[32 * k + 31]);
-          }
-          m_raw = fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
         } else {
           // own 64 columns, and the other half's 64 for the maximum only
           const uint32_t other = static_cast<uint32_t>(kC - col0);
@@ -660,29 +657,38 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
               if (static_cast<int>(other) + c >= src.valid) o[c] = -INFINITY;
             }
           }
-          float mx[4];
+          float mx[2];
 #pragma unroll
           for (int k = 0; k < 2; ++k) {
-            mx[k] = fmax3(s[32 * k], s[32 * k + 1], s[32 * k + 2]);
-            mx[2 + k] = fmax3(o[32 * k], o[32 * k + 1], o[32 * k + 2]);
+            mx[k] = fmax3(o[32 * k], o[32 * k + 1], o[32 * k + 2]);
 #pragma unroll
-            for (int c = 3; c < 31; c += 2) {
-              mx[k] = fmax3(mx[k], s[32 * k + c], s[32 * k + c + 1]);
-              mx[2 + k] = fmax3(mx[2 + k], o[32 * k + c], o[32 * k + c + 1]);
-            }
-            mx[k] = fmaxf(mx[k], s[32 * k + 31]);
-            mx[2 + k] = fmaxf(mx[2 + k], o[32 * k + 31]);
+            for (int c = 3; c < 31; c += 2) mx[k] = fmax3(mx[k], o[32 * k + c], o[32 * k + c + 1]);
+            mx[k] = fmaxf(mx[k], o[32 * k + 31]);
           }
-          m_raw = fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
+          m_other = fmaxf(mx[0], mx[1]);
         }
-        const float m_tile = fmaf(m_raw, c_t, shift);
-        if (j == 0) {
-          m_run = m_tile;
-        } else if (__any_sync(0xffffffffu, m_tile > m_run + 8.0f)) {
-          // O must first hold P_j-1 V_j-1: group G + j + 1 complete
-          if (!wait_group(G + j + 1, 9)) goto softmax_done;
+        // the row maximum of the raw scores: four independent chains of
+        // 3-input max over this thread's columns (and the other half's maximum)
+        auto row_max = [&]() -> float {
+          constexpr int kChains = kC / 32;
+          float mx[kChains];
+#pragma unroll
+          for (int k = 0; k < kChains; ++k) {
+            mx[k] = fmax3(s[32 * k], s[32 * k + 1], s[32 * k + 2]);
+#pragma unroll
+            for (int c = 3; c < 31; c += 2) mx[k] = fmax3(mx[k], s[32 * k + c], s[32 * k + c + 1]);
+            mx[k] = fmaxf(mx[k], s[32 * k + 31]);
+          }
+          if constexpr (kChains == 4)
+            return fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
+          else
+            return fmax3(mx[0], mx[1], m_other);
+        };
+        // rescale this row's O columns and l for a new running maximum m_new (O
+        // must first hold P_j-1 V_j-1: group G + j + 1 complete)
+        auto rescale = [&](float m_new) -> bool {
+          if (!wait_group(G + j + 1, 9)) return false;
           tc_fence_after();
-          const float m_new = fmaxf(m_run, m_tile);
           const float alpha = ex2_approx(m_run - m_new);
           const f32x2 alpha2 = make_f32x2(alpha, alpha);
           m_run = m_new;
@@ -703,56 +709,83 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
             }
             tmem_st16(t_o + 16u * cc, o);
           }
-        }
+          return true;
+        };
         // P = exp2(c * S + shift - m) into P buffer b: bf16 pairs (32 keys = 16
-        // columns at a time), or for a cached tile E4M3 quads (32 keys = 8 columns)
-        const float bias = (kF8 ? shift + wshift : 0.f) - m_run;
-        const f32x2 negm = make_f32x2(bias, bias);
-        const f32x2 c2 = kF8 ? make_f32x2(c_t, c_t) : sl2x2;
+        // columns at a time), or for a cached tile E4M3 quads (32 keys = 8
+        // columns); returns this thread's sum of the weights written
         const uint32_t t_p = tmem + lane_off + kColP + 64u * b;
-        f32x2 lacc[4];
+        auto write_p = [&]() -> float {
+          const float bias = (kF8 ? shift + wshift : 0.f) - m_run;
+          const f32x2 negm = make_f32x2(bias, bias);
+          const f32x2 c2 = kF8 ? make_f32x2(c_t, c_t) : sl2x2;
+          f32x2 lacc[4];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) lacc[i] = make_f32x2(0.f, 0.f);
-        if (t8) {
+          for (int i = 0; i < 4; ++i) lacc[i] = make_f32x2(0.f, 0.f);
+          if (t8) {
 #pragma unroll
-          for (int k = 0; k < kC / 32; ++k) {
-            uint32_t pk[8];
+            for (int k = 0; k < kC / 32; ++k) {
+              uint32_t pk[8];
 #pragma unroll
-            for (int c = 0; c < 8; ++c) {
-              const f32x2 e01 = fma_f32x2(make_f32x2(s[32 * k + 4 * c], s[32 * k + 4 * c + 1]), c2, negm);
-              const f32x2 e23 = fma_f32x2(make_f32x2(s[32 * k + 4 * c + 2], s[32 * k + 4 * c + 3]), c2, negm);
-              float e0, e1, e2, e3;
-              split_f32x2(e01, e0, e1);
-              split_f32x2(e23, e2, e3);
-              const float x0 = ex2_approx(e0), x1 = ex2_approx(e1), x2 = ex2_approx(e2), x3 = ex2_approx(e3);
-              lacc[(2 * c) & 3] = add_f32x2(lacc[(2 * c) & 3], make_f32x2(x0, x1));
-              lacc[(2 * c + 1) & 3] = add_f32x2(lacc[(2 * c + 1) & 3], make_f32x2(x2, x3));
-              pk[c] = pack_e4m3x4(x0, x1, x2, x3);
+              for (int c = 0; c < 8; ++c) {
+                const f32x2 e01 = fma_f32x2(make_f32x2(s[32 * k + 4 * c], s[32 * k + 4 * c + 1]), c2, negm);
+                const f32x2 e23 = fma_f32x2(make_f32x2(s[32 * k + 4 * c + 2], s[32 * k + 4 * c + 3]), c2, negm);
+                float e0, e1, e2, e3;
+                split_f32x2(e01, e0, e1);
+                split_f32x2(e23, e2, e3);
+                const float x0 = ex2_approx(e0), x1 = ex2_approx(e1), x2 = ex2_approx(e2), x3 = ex2_approx(e3);
+                lacc[(2 * c) & 3] = add_f32x2(lacc[(2 * c) & 3], make_f32x2(x0, x1));
+                lacc[(2 * c + 1) & 3] = add_f32x2(lacc[(2 * c + 1) & 3], make_f32x2(x2, x3));
+                pk[c] = pack_e4m3x4(x0, x1, x2, x3);
+              }
+              tmem_st8(t_p + static_cast<uint32_t>(col0 / 4) + 8u * k, pk);
             }
-            tmem_st8(t_p + static_cast<uint32_t>(col0 / 4) + 8u * k, pk);
-          }
-        } else {
+          } else {
 #pragma unroll
-          for (int k = 0; k < kC / 32; ++k) {
-            uint32_t pk[16];
+            for (int k = 0; k < kC / 32; ++k) {
+              uint32_t pk[16];
 #pragma unroll
-            for (int c = 0; c < 16; ++c) {
-              const f32x2 e = fma_f32x2(make_f32x2(s[32 * k + 2 * c], s[32 * k + 2 * c + 1]), c2, negm);
-              float e0, e1;
-              split_f32x2(e, e0, e1);
-              const float x = ex2_approx(e0), y = ex2_approx(e1);
-              lacc[c & 3] = add_f32x2(lacc[c & 3], make_f32x2(x, y));
-              pk[c] = pack_bf16x2(x, y);
+              for (int c = 0; c < 16; ++c) {
+                const f32x2 e = fma_f32x2(make_f32x2(s[32 * k + 2 * c], s[32 * k + 2 * c + 1]), c2, negm);
+                float e0, e1;
+                split_f32x2(e, e0, e1);
+                const float x = ex2_approx(e0), y = ex2_approx(e1);
+                lacc[c & 3] = add_f32x2(lacc[c & 3], make_f32x2(x, y));
+                pk[c] = pack_bf16x2(x, y);
+              }
+              tmem_st16(t_p + static_cast<uint32_t>(col0 / 2) + 16u * k, pk);
             }
-            tmem_st16(t_p + static_cast<uint32_t>(col0 / 2) + 16u * k, pk);
           }
-        }
-        {
           const f32x2 l2 = add_f32x2(add_f32x2(lacc[0], lacc[1]), add_f32x2(lacc[2], lacc[3]));
           float lo, hi;
           split_f32x2(l2, lo, hi);
-          l_run += kF8 ? (lo + hi) * lscale : lo + hi;
+          return lo + hi;
+        };
+        float l_tile;
+        if (!kMaxFree || j == 0) {
+          // running maximum from the row maximum (lazy: moves only when a tile's
+          // maximum exceeds it by more than 2^8)
+          const float m_tile = fmaf(row_max(), c_t, shift);
+          if (j == 0) {
+            m_run = m_tile;
+          } else if (__any_sync(0xffffffffu, m_tile > m_run + 8.0f)) {
+            if (!rescale(fmaxf(m_run, m_tile))) goto softmax_done;
+          }
+          l_tile = write_p();
+        } else {
+          // exponentials against the current maximum, checked by their sum: a
+          // sum within kWeightLimit bounds every weight (E4M3 weights at most
+          // 448, bf16 weights far from fp32 overflow); otherwise take the row
+          // maximum, rescale, and write P again
+          l_tile = write_p();
+          const float limit = t8 ? 448.f : 1.8446744e19f;  // 448, 2^64
+          if (__any_sync(0xffffffffu, !(l_tile <= limit))) {
+            const float m_tile = fmaf(row_max(), c_t, shift);
+            if (!rescale(fmaxf(m_run, m_tile))) goto softmax_done;
+            l_tile = write_p();
+          }
         }
+        l_run += kF8 ? l_tile * lscale : l_tile;
         // the MMA thread waits only for P: the leader's warp 0 first makes
         // sure that the stage of P_j V_j's group (G + j + 2) has landed
         if (leader && warp == 0 &&

@@ -271,3 +271,24 @@ def test_call_launch_counts():
     rcb.set_kernel("tcgen05")
     tiny = rcb.RefCache(rcb.Segments.from_workload(workloads.TINY), num_layers=1, mask_mode="beyond")
     assert tiny.launches("step") == 1 and tiny.launches("build") == 2
+
+
+def _growing_keys(w, growth=0.5):
+    """Seeded inputs whose cached keys grow tile by tile (rows of key tile t of
+    R scaled by 1 + growth * t), so that a row's running maximum rises by more
+    than 2^8 several times after its first tile and the rescale path runs."""
+    qs, ks, vs = workloads.static_qkv(w)
+    ks = ks.float()
+    for b, r in enumerate(w.requests):
+        r0 = w.cu_static[b] + r.n_st
+        t = torch.arange(r.n_r, dtype=torch.float32) // 128
+        ks[r0:r0 + r.n_r] *= (1.0 + growth * t)[:, None, None]
+    return qs, ks.to(torch.bfloat16), vs
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("head_dim", [64, 128])
+def test_rescale_path_full_compare(kernel, head_dim):
+    w = workloads.Workload(f"growing_keys_d{head_dim}", 2, head_dim, (workloads.Request(16, 32, 200, 1500),), 13)
+    run = pu.GpuRun(w, kernel=kernel, static=_growing_keys(w))
+    pu.full_compare(run)
