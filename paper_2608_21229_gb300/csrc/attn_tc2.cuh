@@ -78,9 +78,6 @@
 // at most 2^8; each tile adds its unshifted weight sum to l, and
 // O = s_ref * acc / l.
 #pragma once
-#ifndef RC_SOFTMAX_MAXFREE
-#define RC_SOFTMAX_MAXFREE 0
-#endif
 #include "attn_tc.cuh"
 
 namespace rc {
@@ -490,9 +487,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
     // epilogue through shared memory.
     constexpr int kH = Cfg::kHalves;
     constexpr int kC = 128 / kH;  // key columns and O columns of this thread
-    // one softmax thread per row: after a row's first tile, exponentials are
-    // taken against the running maximum and checked by their sum
-    constexpr bool kMaxFree = kH == 1 && RC_SOFTMAX_MAXFREE;
     const int quarter = warp & 3, hh = warp >> 2;
     const int col0 = hh * kC;
     const int trow = quarter * 32 + lane;                  // row within this CTA's 128 rows (= TMEM lane)
@@ -761,30 +755,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
           split_f32x2(l2, lo, hi);
           return lo + hi;
         };
-        float l_tile;
-        if (!kMaxFree || j == 0) {
-          // running maximum from the row maximum (lazy: moves only when a tile's
-          // maximum exceeds it by more than 2^8)
-          const float m_tile = fmaf(row_max(), c_t, shift);
-          if (j == 0) {
-            m_run = m_tile;
-          } else if (__any_sync(0xffffffffu, m_tile > m_run + 8.0f)) {
-            if (!rescale(fmaxf(m_run, m_tile))) goto softmax_done;
-          }
-          l_tile = write_p();
-        } else {
-          // exponentials against the current maximum, checked by their sum: a
-          // sum within kWeightLimit bounds every weight (E4M3 weights at most
-          // 448, bf16 weights far from fp32 overflow); otherwise take the row
-          // maximum, rescale, and write P again
-          l_tile = write_p();
-          const float limit = t8 ? 448.f : 1.8446744e19f;  // 448, 2^64
-          if (__any_sync(0xffffffffu, !(l_tile <= limit))) {
-            const float m_tile = fmaf(row_max(), c_t, shift);
-            if (!rescale(fmaxf(m_run, m_tile))) goto softmax_done;
-            l_tile = write_p();
-          }
+        // running maximum from the row maximum (lazy: moves only when a tile's
+        // maximum exceeds it by more than 2^8)
+        const float m_tile = fmaf(row_max(), c_t, shift);
+        if (j == 0) {
+          m_run = m_tile;
+        } else if (__any_sync(0xffffffffu, m_tile > m_run + 8.0f)) {
+          if (!rescale(fmaxf(m_run, m_tile))) goto softmax_done;
         }
+        const float l_tile = write_p();
         l_run += kF8 ? l_tile * lscale : l_tile;
         // the MMA thread waits only for P: the leader's warp 0 first makes
         // sure that the stage of P_j V_j's group (G + j + 2) has landed
