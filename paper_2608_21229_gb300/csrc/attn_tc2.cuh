@@ -13,7 +13,8 @@
 // CTA keeps its own 128 query rows (A is split along M).  Per SM this halves
 // the tile bytes fetched and the B-operand bytes read, for the same MMA work.
 //
-// Cluster of 2 CTAs (rank 0 = leader), 224 threads each:
+// Cluster of 2 CTAs (rank 0 = leader), 224 threads each (352 in the E4M3
+// kernel, whose 8 softmax warps split each row's columns, see below):
 //   warps 0-3  softmax: thread l of warp w owns row 32 w + l of this CTA's
 //              128 rows (its TMEM lane), all 128 score columns of a tile
 //   warp 4     TMA producer: this CTA's Q rows and its halves of the K and V
@@ -69,8 +70,10 @@
 // start of an item with cached tiles every softmax thread quantises its own
 // query row of this head into an E4M3 Q tile (one scale per row), and the
 // first cached tile's S waits for it (q8_full, one arrival per softmax warp
-// of both CTAs).  The
-// scales enter the softmax, so one O accumulator serves both ranges: with
+// of both CTAs).  The producer also feeds each CTA a small shared-memory ring
+// of the cached tiles' scales (16-byte bulk copies), so that the softmax loop
+// touches no global memory.  The scales enter the softmax, so one O
+// accumulator serves both ranges: with
 // s_ref = s_V of the item's first cached tile, the weights written are
 //   live tile:    exp2(u - m) / s_ref                   (bf16, u = scaled score)
 //   cached tile:  exp2(u + delta - m), delta = log2(s_V / s_ref)   (E4M3)
