@@ -1,7 +1,10 @@
 // refcache.cu -- the C ABI declared in include/refcache.h: argument checks,
-// the per-request work tables, the persistent per-layer K/V cache, TMA tensor
-// maps and the kernel launches.  All compute runs in the kernels of
-// attn_tc.cuh (default) or attn_mma.cuh.
+// the per-request work tables, the persistent per-layer K/V cache (bf16, or
+// E4M3 with REFCACHE_CACHE_FP8), TMA tensor maps and the kernel launches.  All
+// compute runs in the kernels of attn_tc2.cuh (head dim 128, CTA pairs),
+// attn_tc.cuh (head dim 64), attn_mma.cuh (the mma.sync comparison kernel and
+// the cache copy), attn_combine.cuh (merge of split items) and cache_fp8.cuh
+// (the E4M3 cache write).
 #include <cuda.h>
 #include <cuda_runtime.h>
 
