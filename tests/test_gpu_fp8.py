@@ -250,3 +250,23 @@ def test_fp8_rescale_path_full_compare():
     # tiles carry the weight), so the rounding of those weights does not
     # average out: only the worst-case bound applies
     check_step(run, heads=[0, 1], statistical=False)
+
+
+def test_accessors_refuse_the_other_cache_format():
+    w = workloads.CFG_SMALL
+    seg = rcb.Segments.from_workload(w)
+    c8 = rcb.RefCache(seg, device="cuda:0", cache_dtype="fp8")
+    c16 = rcb.RefCache(seg, device="cuda:0")
+    with pytest.raises(rcb.RefCacheError) as e:
+        c8.kv(0)
+    assert e.value.code == rcb.ERR_UNSUPPORTED
+    with pytest.raises(rcb.RefCacheError) as e:
+        c16.fp8(0)
+    assert e.value.code == rcb.ERR_UNSUPPORTED
+    with pytest.raises(rcb.RefCacheError) as e:
+        c8.fp8(1)  # one layer only
+    assert e.value.code == rcb.ERR_INVALID_ARG
+    k8, vt8, sc = c8.fp8(0)
+    rows_pad = sum((r.n_r + 127) // 128 * 128 for r in w.requests)
+    assert k8.shape == (rows_pad, w.num_heads, w.head_dim) and vt8.shape == (w.num_heads, w.head_dim, rows_pad)
+    assert sc.shape == (rows_pad // 128, w.num_heads, 4)
