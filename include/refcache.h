@@ -47,6 +47,11 @@
  *   - The refcache_build and step_attention calls of one cache share that
  *     workspace: issue them in stream order (one stream, or streams ordered
  *     by events), not concurrently.
+ *   - refcache_build and step_attention only launch kernels (no allocation,
+ *     no copy), so they can be captured in a CUDA graph and replayed, once a
+ *     first call on the device has run outside the capture (the kernels'
+ *     attributes are set on first use).  full_attention is not capturable
+ *     (it copies its work list from host memory).
  */
 #ifndef REFCACHE_H
 #define REFCACHE_H
