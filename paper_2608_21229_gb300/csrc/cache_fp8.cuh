@@ -40,66 +40,71 @@ __device__ __forceinline__ float block_amax_256(float v, float* red) {
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
-// grid (tiles, H), 256 threads: thread i holds row (i >> 4) + 16 r, columns
-// [8 (i & 15), 8 (i & 15) + 8) of the tile, r = 0..7.
-__global__ void __launch_bounds__(256) quantize_cache_kernel(const QuantTile* __restrict__ tiles,
-                                                             const uint4* __restrict__ k, const uint4* __restrict__ v,
-                                                             uint8_t* __restrict__ k8, uint8_t* __restrict__ vt8,
-                                                             float4* __restrict__ scales, int H, int64_t rows_pad) {
+// grid (H, tiles, 2): blockIdx.z = 0 quantises the tile's K, 1 its V (heads
+// fastest, so that CTAs running together read neighbouring bytes of the same
+// rows); 256 threads.  Thread i takes rows [4 q, 4 q + 4) of the tile (q = i % 32) and
+// head-dim columns [16 p, 16 p + 16) (p = i / 32): per row one 32-byte run.
+// K codes go out row by row (16 bytes); V codes are transposed through shared
+// memory as one 32-bit word (four rows) per column, so the 32 threads of a
+// warp store 32 consecutive words.
+__global__ void __launch_bounds__(256, 3) quantize_cache_kernel(const QuantTile* __restrict__ tiles,
+                                                                const uint4* __restrict__ k, const uint4* __restrict__ v,
+                                                                uint8_t* __restrict__ k8, uint8_t* __restrict__ vt8,
+                                                                float4* __restrict__ scales, int H, int64_t rows_pad) {
   constexpr int D = 128;
-  __shared__ float red[2][8];
-  __shared__ __align__(16) uint8_t vt[D][128 + 16];  // V^T codes of the tile: [d][row]
-  const QuantTile t = tiles[blockIdx.x];
-  const int h = blockIdx.y;
-  const int c = threadIdx.x & 15;
-  const int r0 = threadIdx.x >> 4;
+  __shared__ float red[8];
+  __shared__ __align__(16) uint32_t vt[D][32 + 4];  // V^T codes of the tile: [d][row / 4], 4 rows per word
+  const QuantTile t = tiles[blockIdx.y];
+  const int h = blockIdx.x;
+  const bool is_v = blockIdx.z != 0;
+  const int q = threadIdx.x & 31;   // rows 4 q .. 4 q + 3
+  const int p = threadIdx.x >> 5;   // columns 16 p .. 16 p + 15
   const int64_t row_u4 = static_cast<int64_t>(H) * D / 8;
-  uint4 kv[8], vv[8];
-  float ka = 0.f, va = 0.f;
+  const uint4* src = is_v ? v : k;
+  uint4 x[4][2];
+  float a = 0.f;
 #pragma unroll
-  for (int r = 0; r < 8; ++r) {
-    const int row = r0 + 16 * r;
-    if (row < t.valid) {
-      const int64_t at = static_cast<int64_t>(t.src_row0 + row) * row_u4 + h * (D / 8) + c;
-      kv[r] = k[at];
-      vv[r] = v[at];
-    } else {
-      kv[r] = make_uint4(0, 0, 0, 0);
-      vv[r] = make_uint4(0, 0, 0, 0);
-    }
-    const uint32_t kw[4] = {kv[r].x, kv[r].y, kv[r].z, kv[r].w};
-    const uint32_t vw[4] = {vv[r].x, vv[r].y, vv[r].z, vv[r].w};
+  for (int r = 0; r < 4; ++r) {
+    const int row = 4 * q + r;
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      ka = fmax3(ka, fabsf(bf16_lo(kw[e])), fabsf(bf16_hi(kw[e])));
-      va = fmax3(va, fabsf(bf16_lo(vw[e])), fabsf(bf16_hi(vw[e])));
+    for (int c = 0; c < 2; ++c) {
+      x[r][c] = row < t.valid ? src[static_cast<int64_t>(t.src_row0 + row) * row_u4 + h * (D / 8) + 2 * p + c]
+                              : make_uint4(0, 0, 0, 0);
+      const uint32_t w[4] = {x[r][c].x, x[r][c].y, x[r][c].z, x[r][c].w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) a = fmax3(a, fabsf(bf16_lo(w[e])), fabsf(bf16_hi(w[e])));
     }
   }
-  const float kmax = block_amax_256(ka, red[0]);
-  const float vmax = block_amax_256(va, red[1]);
-  const float kinv = kmax > 0.f ? __fdiv_rn(448.f, kmax) : 0.f;
-  const float vinv = vmax > 0.f ? __fdiv_rn(448.f, vmax) : 0.f;
-  uint8_t* krow = k8 + static_cast<int64_t>(t.dst_row0) * H * D + static_cast<int64_t>(h) * D + 8 * c;
+  const float amax = block_amax_256(a, red);
+  const float inv = amax > 0.f ? __fdiv_rn(448.f, amax) : 0.f;
+  // codes of the 16 columns of row r: four words of four codes
+  uint32_t cw[4][4];
 #pragma unroll
-  for (int r = 0; r < 8; ++r) {
-    const int row = r0 + 16 * r;
-    const uint32_t kw[4] = {kv[r].x, kv[r].y, kv[r].z, kv[r].w};
-    const uint32_t vw[4] = {vv[r].x, vv[r].y, vv[r].z, vv[r].w};
-    const uint32_t k_lo = pack_e4m3x4(__fmul_rn(bf16_lo(kw[0]), kinv), __fmul_rn(bf16_hi(kw[0]), kinv),
-                                      __fmul_rn(bf16_lo(kw[1]), kinv), __fmul_rn(bf16_hi(kw[1]), kinv));
-    const uint32_t k_hi = pack_e4m3x4(__fmul_rn(bf16_lo(kw[2]), kinv), __fmul_rn(bf16_hi(kw[2]), kinv),
-                                      __fmul_rn(bf16_lo(kw[3]), kinv), __fmul_rn(bf16_hi(kw[3]), kinv));
-    *reinterpret_cast<uint2*>(krow + static_cast<int64_t>(row) * H * D) = make_uint2(k_lo, k_hi);
-    const uint32_t v_lo = pack_e4m3x4(__fmul_rn(bf16_lo(vw[0]), vinv), __fmul_rn(bf16_hi(vw[0]), vinv),
-                                      __fmul_rn(bf16_lo(vw[1]), vinv), __fmul_rn(bf16_hi(vw[1]), vinv));
-    const uint32_t v_hi = pack_e4m3x4(__fmul_rn(bf16_lo(vw[2]), vinv), __fmul_rn(bf16_hi(vw[2]), vinv),
-                                      __fmul_rn(bf16_lo(vw[3]), vinv), __fmul_rn(bf16_hi(vw[3]), vinv));
+  for (int r = 0; r < 4; ++r)
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      vt[8 * c + e][row] = static_cast<uint8_t>(v_lo >> (8 * e));
-      vt[8 * c + 4 + e][row] = static_cast<uint8_t>(v_hi >> (8 * e));
+    for (int c = 0; c < 2; ++c) {
+      const uint4& y = x[r][c];
+      cw[r][2 * c] = pack_e4m3x4(__fmul_rn(bf16_lo(y.x), inv), __fmul_rn(bf16_hi(y.x), inv),
+                                 __fmul_rn(bf16_lo(y.y), inv), __fmul_rn(bf16_hi(y.y), inv));
+      cw[r][2 * c + 1] = pack_e4m3x4(__fmul_rn(bf16_lo(y.z), inv), __fmul_rn(bf16_hi(y.z), inv),
+                                     __fmul_rn(bf16_lo(y.w), inv), __fmul_rn(bf16_hi(y.w), inv));
     }
+  if (!is_v) {
+    uint8_t* krow = k8 + static_cast<int64_t>(t.dst_row0) * H * D + static_cast<int64_t>(h) * D + 16 * p;
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+      *reinterpret_cast<uint4*>(krow + static_cast<int64_t>(4 * q + r) * H * D) =
+          make_uint4(cw[r][0], cw[r][1], cw[r][2], cw[r][3]);
+    if (threadIdx.x == 0) scales[static_cast<int64_t>(t.dst_row0 >> 7) * H + h].x = __fdiv_rn(amax, 448.f);
+    return;
   }
+  // column 16 p + 4 w + e: byte e of word w of each of the four rows
+#pragma unroll
+  for (int w = 0; w < 4; ++w)
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+      vt[16 * p + 4 * w + e][q] = __byte_perm(__byte_perm(cw[0][w], cw[1][w], 0x0040 + e * 0x0011),
+                                              __byte_perm(cw[2][w], cw[3][w], 0x0040 + e * 0x0011), 0x5410);
   __syncthreads();
   // V^T rows: 128 d rows of 128 codes, 16 bytes per thread and step
   uint8_t* vbase = vt8 + static_cast<int64_t>(h) * D * rows_pad + t.dst_row0;
@@ -108,12 +113,14 @@ __global__ void __launch_bounds__(256) quantize_cache_kernel(const QuantTile* __
     const int idx = threadIdx.x + 256 * i;  // 0..1023 = d * 8 + chunk
     const int d = idx >> 3, ch = idx & 7;
     *reinterpret_cast<uint4*>(vbase + static_cast<int64_t>(d) * rows_pad + 16 * ch) =
-        *reinterpret_cast<const uint4*>(&vt[d][16 * ch]);
+        *reinterpret_cast<const uint4*>(&vt[d][4 * ch]);
   }
   if (threadIdx.x == 0) {
-    const float sv = __fdiv_rn(vmax, 448.f);
-    scales[static_cast<int64_t>(t.dst_row0 >> 7) * H + h] =
-        make_float4(__fdiv_rn(kmax, 448.f), sv, sv > 0.f ? log2f(sv) : 0.f, sv > 0.f ? __frcp_rn(sv) : 0.f);
+    const float sv = __fdiv_rn(amax, 448.f);
+    float4* dst = &scales[static_cast<int64_t>(t.dst_row0 >> 7) * H + h];
+    dst->y = sv;
+    dst->z = sv > 0.f ? log2f(sv) : 0.f;
+    dst->w = sv > 0.f ? __frcp_rn(sv) : 0.f;
   }
 }
 

@@ -815,7 +815,7 @@ int refcache_build(refcache_t* h, int layer, const void* q_static, const void* k
   if (h->f8 && h->n_qtiles > 0) {
     void *k8 = nullptr, *vt8 = nullptr, *sc = nullptr;
     refcache_fp8_ptr(h, layer, &k8, &vt8, &sc, nullptr);
-    rc::quantize_cache_kernel<<<dim3(static_cast<unsigned>(h->n_qtiles), static_cast<unsigned>(h->H)), 256, 0, s>>>(
+    rc::quantize_cache_kernel<<<dim3(static_cast<unsigned>(h->H), static_cast<unsigned>(h->n_qtiles), 2), 256, 0, s>>>(
         h->d_qtiles, static_cast<const uint4*>(k_static), static_cast<const uint4*>(v_static),
         static_cast<uint8_t*>(k8), static_cast<uint8_t*>(vt8), static_cast<float4*>(sc), h->H, h->rows_pad);
     cudaError_t e = cudaGetLastError();
