@@ -270,3 +270,10 @@ def test_accessors_refuse_the_other_cache_format():
     rows_pad = sum((r.n_r + 127) // 128 * 128 for r in w.requests)
     assert k8.shape == (rows_pad, w.num_heads, w.head_dim) and vt8.shape == (w.num_heads, w.head_dim, rows_pad)
     assert sc.shape == (rows_pad // 128, w.num_heads, 4)
+
+
+def test_fp8_ragged_4req_sampled():
+    """The paper-shaped ragged serving batch (four requests, 1 to 8 references)
+    on the E4M3 cache, sampled at full size."""
+    run = Fp8Run(workloads.RAGGED_4REQ)
+    check_step(run, heads=[2, 19], rows_per_request=24, seed=11)
