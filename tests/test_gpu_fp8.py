@@ -277,3 +277,15 @@ def test_fp8_ragged_4req_sampled():
     on the E4M3 cache, sampled at full size."""
     run = Fp8Run(workloads.RAGGED_4REQ)
     check_step(run, heads=[2, 19], rows_per_request=24, seed=11)
+
+
+@pytest.mark.parametrize("seed", [31, 32, 33])
+def test_fp8_many_ragged_requests(seed):
+    """Up to a dozen ragged requests per batch (empty and one-row segments,
+    caches across tile edges), every output of two heads against the oracle."""
+    rng = np.random.default_rng(seed)
+    reqs = list(workloads.random_requests(rng, int(rng.integers(6, 12)), max_len=300))
+    reqs.append(workloads.Request(0, 0, 1, 1))
+    w = workloads.Workload(f"fp8_many_{seed}", 3, 128, tuple(reqs), seed)
+    run = Fp8Run(w)
+    check_step(run, heads=[0, 2])
