@@ -104,6 +104,12 @@ class ClockSampler:
                  "-lms", "200"], stdout=self.tmp, stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
+            return self
+        # nvidia-smi's start-up holds up kernel launches for a few milliseconds:
+        # let it write its first sample before the timed region begins
+        t_end = time.monotonic() + 5.0
+        while time.monotonic() < t_end and self.proc.poll() is None and os.path.getsize(self.tmp.name) == 0:
+            time.sleep(0.01)
         return self
 
     def __exit__(self, *exc):
