@@ -657,16 +657,22 @@ def run_e2e(args, w, cache, seg, dev, stream, scale, flops_per_step):
 
     one()
     torch.cuda.synchronize()
-    n = max(1, min(args.steps, 3))
-    a, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    a.record(stream)
-    for _ in range(n):
-        one()
-    b_.record(stream)  # after the last copies out (the stream waited for them)
-    torch.cuda.synchronize()
-    secs = a.elapsed_time(b_) / 1e3 / n
+    # each step timed on its own (events after the stream has waited for the
+    # last copies out); the value is the median step, so that a stray slow
+    # step (the host is shared) does not decide it -- every step is listed
+    n = max(5, min(args.steps, 7))
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        for a, b_ in evs:
+            a.record(stream)
+            one()
+            b_.record(stream)
+        torch.cuda.synchronize()
+    ms = [a.elapsed_time(b_) for a, b_ in evs]
+    secs = statistics.median(ms) / 1e3
     return {"value": flops_per_step / secs / 1e12, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-            "ms_per_step": secs * 1e3, "steps": n,
+            "ms_per_step": secs * 1e3, "steps": n, "timing": "median of the steps",
+            "step_ms": [round(x, 3) for x in ms], "mean_ms": statistics.mean(ms), "clocks": clk.summary(),
             "overlap": "copies in on a copy stream (2 device buffers), copies out on a third stream, "
                        "ordered by events; every byte moves inside the timed region"}
 
