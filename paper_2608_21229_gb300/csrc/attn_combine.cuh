@@ -13,6 +13,7 @@
 #include <cuda_bf16.h>
 
 #include "common.cuh"
+#include "ptx.cuh"
 
 namespace rc {
 
@@ -27,6 +28,8 @@ __global__ void __launch_bounds__(256) combine_parts_kernel(const CombineJob* __
                                                             __nv_bfloat16* __restrict__ out, float* __restrict__ lse,
                                                             int64_t row_stride, int num_heads) {
   static_assert(D == 128, "four columns per lane");
+  grid_dependency_wait();  // the attention kernel's parts are complete
+  if (threadIdx.x == 0) grid_launch_dependents();
   const CombineJob job = jobs[blockIdx.y];
   const int r = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (r >= job.q_rows) return;

@@ -230,6 +230,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
   __syncthreads();
   cluster_sync();  // both CTAs' barriers exist before any cross-CTA arrival
   tc_fence_after();
+  // launched as a programmatic dependent of the previous kernel on the stream:
+  // everything above overlaps its tail, nothing below reads memory before it
+  // is complete; and the next kernel may start its CTAs (they wait likewise)
+  grid_dependency_wait();
+  if (threadIdx.x == 0) grid_launch_dependents();
   const uint32_t tmem = *tmem_holder;
   const Ctl ctl{abort_flag, args.timeout_ns};
   auto lbar = [&](int i) -> uint32_t { return mapa_shared(bar(i), 0); };  // leader's barrier i

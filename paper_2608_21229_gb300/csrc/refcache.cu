@@ -246,9 +246,20 @@ int launch_tc2(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info
   int rc = tc2_clusters<kF8>(info, &max_clusters);
   if (rc) return rc;
   const int clusters = std::min(a.n_items, max_clusters);
-  rc::attn_tc2_kernel<kF8>
-      <<<2 * clusters, rc::tc2::Cfg<kF8>::kThreads, smem, s>>>(maps[0], maps[1], maps[2], maps[3], maps[4], a);
-  cudaError_t e = cudaGetLastError();
+  // a programmatic dependent of the stream's previous kernel: its prologue
+  // (barriers, tensor memory) overlaps that kernel's tail
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(2 * static_cast<unsigned>(clusters), 1, 1);
+  cfg.blockDim = dim3(rc::tc2::Cfg<kF8>::kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, rc::attn_tc2_kernel<kF8>, maps[0], maps[1], maps[2], maps[3], maps[4], a);
+  if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "attn_tc2_kernel launch");
   return REFCACHE_OK;
 }
@@ -352,10 +363,19 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
   }
   if ((rc = f8 ? launch_tc2<true>(maps, a, info, s) : launch_tc2<false>(maps, a, info, s)) != 0) return rc;
   if (il && il->n_jobs > 0) {
-    const dim3 grid(static_cast<unsigned>((a.rows_per_task + 7) / 8), static_cast<unsigned>(il->n_jobs));
-    rc::combine_parts_kernel<128><<<grid, 256, 0, s>>>(il->jobs, il->part_o, il->part_lse, a.rows_per_task, a.out,
-                                                       a.lse, a.row_stride, H);
-    cudaError_t e = cudaGetLastError();
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(static_cast<unsigned>((a.rows_per_task + 7) / 8), static_cast<unsigned>(il->n_jobs));
+    cfg.blockDim = dim3(256, 1, 1);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;  // its CTAs wait for the attention kernel
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, rc::combine_parts_kernel<128>, il->jobs,
+                                       static_cast<const float*>(il->part_o), static_cast<const float*>(il->part_lse),
+                                       a.rows_per_task, a.out, a.lse, a.row_stride, H);
+    if (e == cudaSuccess) e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "combine_parts_kernel launch");
   }
   return REFCACHE_OK;
