@@ -47,6 +47,13 @@
  *   - The refcache_build and step_attention calls of one cache share that
  *     workspace: issue them in stream order (one stream, or streams ordered
  *     by events), not concurrently.
+ *   - The head-dim-128 attention kernel and the merge of split items are
+ *     launched as programmatic dependents of the previous kernel on the
+ *     stream: they wait for it to complete before they read memory, and they
+ *     allow the kernel after them to start early.  A caller's kernel launched
+ *     with programmatic stream serialization after a library call must
+ *     therefore wait for its grid dependencies (griddepcontrol.wait) before it
+ *     reads the library's outputs; ordinary launches need nothing.
  *   - refcache_build and step_attention only launch kernels (no allocation,
  *     no copy), so they can be captured in a CUDA graph and replayed, once a
  *     first call on the device has run outside the capture (the kernels'
