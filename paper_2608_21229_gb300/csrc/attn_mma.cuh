@@ -11,6 +11,7 @@
 #include <cuda_bf16.h>
 
 #include "common.cuh"
+#include "ptx.cuh"
 
 namespace rc {
 
@@ -226,13 +227,19 @@ __global__ void __launch_bounds__(128) attn_mma_kernel(const AttnArgs a) {
 }
 
 // Cache write (the copy of the static pass's R rows' K and V into the
-// persistent slot of one layer).  One block row per request segment.
+// persistent slot of one layer).  One block row per request segment.  It reads
+// only the static inputs, so it may run beside the prefill attention: launched
+// as a programmatic dependent of that kernel it starts once the prefill's CTAs
+// are all running (and so the inputs' producers are complete), and it waits
+// for the prefill to complete before it exits, so that the work after it on
+// the stream sees both.
 struct CopySeg {
   int32_t src_row0, dst_row0, nrows, pad;
 };
 __global__ void copy_rows_kernel(const CopySeg* segs, const uint4* __restrict__ src_k,
                                  const uint4* __restrict__ src_v, uint4* __restrict__ dst_k,
                                  uint4* __restrict__ dst_v, int row_u4) {
+  if (threadIdx.x == 0) grid_launch_dependents();
   const CopySeg s = segs[blockIdx.y];
   const int64_t n = static_cast<int64_t>(s.nrows) * row_u4;
   const int64_t so = static_cast<int64_t>(s.src_row0) * row_u4, d0 = static_cast<int64_t>(s.dst_row0) * row_u4;
@@ -241,6 +248,7 @@ __global__ void copy_rows_kernel(const CopySeg* segs, const uint4* __restrict__ 
     dst_k[d0 + i] = src_k[so + i];
     dst_v[d0 + i] = src_v[so + i];
   }
+  grid_dependency_wait();
 }
 
 }  // namespace rc

@@ -310,9 +310,46 @@ struct ItemList {
   float* part_lse = nullptr;
 };
 
+// The build's cache write: copy_rows_kernel over the request segments.
+struct CopyJob {
+  const CopySeg* segs = nullptr;
+  int n_segs = 0;
+  const void *src_k = nullptr, *src_v = nullptr;
+  void *dst_k = nullptr, *dst_v = nullptr;
+  int row_u4 = 0;
+  int64_t rows = 0;
+};
+
+// `beside`: launched as a programmatic dependent of the kernel before it, so
+// that it runs next to that kernel (its grid is kept to two CTAs per SM, which
+// fit beside the attention kernel's CTAs).
+int launch_copy(const CopyJob& c, const DeviceInfo* info, cudaStream_t s, bool beside) {
+  const int64_t per_seg = beside ? std::max(1, 2 * info->num_sms / c.n_segs) : 1024;
+  dim3 grid(static_cast<unsigned>(std::min<int64_t>(per_seg, (c.rows * c.row_u4 + 255) / 256 / c.n_segs + 1)),
+            static_cast<unsigned>(c.n_segs));
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(256, 1, 1);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = beside ? 1 : 0;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, rc::copy_rows_kernel, c.segs, static_cast<const uint4*>(c.src_k),
+                                     static_cast<const uint4*>(c.src_v), static_cast<uint4*>(c.dst_k),
+                                     static_cast<uint4*>(c.dst_v), c.row_u4);
+  if (e == cudaSuccess) e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "copy_rows_kernel launch");
+  return REFCACHE_OK;
+}
+
+// `copy` (the build's cache write, if any) runs beside the head-dim-128 pair
+// kernel, launched right after it; with the other kernels it goes first.
 int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands& op, float scale, DeviceInfo* info,
-                  cudaStream_t s, const ItemList* il = nullptr, const Fp8B* f8 = nullptr) {
-  if (n_tasks == 0) return REFCACHE_OK;
+                  cudaStream_t s, const ItemList* il = nullptr, const Fp8B* f8 = nullptr,
+                  const CopyJob* copy = nullptr) {
+  if (n_tasks == 0) return copy ? launch_copy(*copy, info, s, false) : REFCACHE_OK;
   AttnArgs a{};
   a.tasks = d_tasks;
   a.n_tasks = n_tasks;
@@ -332,6 +369,8 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
   if (static_cast<int64_t>(n_tasks) * H > (1ll << 30)) return fail(REFCACHE_ERR_INVALID_ARG, "too many work items");
   if (g_kernel.load() == REFCACHE_KERNEL_MMA_SYNC) {
     if (f8) return fail(REFCACHE_ERR_UNSUPPORTED, "the E4M3 cache runs on the tcgen05 kernel only");
+    int rc = copy ? launch_copy(*copy, info, s, false) : REFCACHE_OK;
+    if (rc) return rc;
     return D == 64 ? launch_mma<64>(a, info, s) : launch_mma<128>(a, info, s);
   }
   // K tiles of the CTA-pair kernel are loaded as two 64-row halves
@@ -353,7 +392,10 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
     maps[4] = maps[2];
   }
   a.dbg_skip_first_load = g_dbg_skip.exchange(0);
-  if (D == 64) return launch_tc<64>(maps, a, info, s);
+  if (D == 64) {
+    if (copy && (rc = launch_copy(*copy, info, s, false)) != 0) return rc;
+    return launch_tc<64>(maps, a, info, s);
+  }
   if (il && il->items) {
     a.tasks = il->items;
     a.per_item = 1;
@@ -362,6 +404,7 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
     a.part_lse = il->part_lse;
   }
   if ((rc = f8 ? launch_tc2<true>(maps, a, info, s) : launch_tc2<false>(maps, a, info, s)) != 0) return rc;
+  if (copy && (rc = launch_copy(*copy, info, s, true)) != 0) return rc;
   if (il && il->n_jobs > 0) {
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3(static_cast<unsigned>((a.rows_per_task + 7) / 8), static_cast<unsigned>(il->n_jobs));
@@ -843,19 +886,20 @@ int refcache_build(refcache_t* h, int layer, const void* q_static, const void* k
   }
   void *kslot = nullptr, *vslot = nullptr;
   if (!h->f8) refcache_kv_ptr(h, layer, &kslot, &vslot, nullptr);
+  CopyJob cj;
   if (h->n_copy > 0) {
-    const int row_u4 = h->H * h->D * 2 / 16;
-    dim3 grid(static_cast<unsigned>(std::min<int64_t>(1024, (h->cache_rows * row_u4 + 255) / 256 / h->n_copy + 1)),
-              static_cast<unsigned>(h->n_copy));
-    rc::copy_rows_kernel<<<grid, 256, 0, s>>>(h->d_copy, static_cast<const uint4*>(k_static),
-                                              static_cast<const uint4*>(v_static), static_cast<uint4*>(kslot),
-                                              static_cast<uint4*>(vslot), row_u4);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return cuda_fail(e, "copy_rows_kernel launch");
+    cj.segs = h->d_copy;
+    cj.n_segs = h->n_copy;
+    cj.src_k = k_static;
+    cj.src_v = v_static;
+    cj.dst_k = kslot;
+    cj.dst_v = vslot;
+    cj.row_u4 = h->H * h->D * 2 / 16;
+    cj.rows = h->cache_rows;
   }
   Operands op{q_static, h->static_rows, k_static, v_static, h->static_rows, nullptr, nullptr, 0, o_static, lse_static};
   rc = run_attention(h->d_build, h->n_build, h->H, h->D, op, softmax_scale, info, s,
-                     h->build_items.items ? &h->build_items : nullptr);
+                     h->build_items.items ? &h->build_items : nullptr, nullptr, h->n_copy > 0 ? &cj : nullptr);
   if (rc) return rc;
   h->built[layer] = 1;
   return REFCACHE_OK;
