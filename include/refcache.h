@@ -157,12 +157,16 @@ REFCACHE_API size_t refcache_bytes(int num_layers, int mask_mode, const refcache
  * the caller, not freed).  Synchronous.  *out is set only on success.
  *
  * For head_dim 128 it also plans, for the current device, the per-item work
- * lists of the prefill and the step: when their (query tile, head) items do
- * not fill the last round of the GPU's CTA pairs evenly, the items of that
- * round are split by key range into 2-8 parts whose outputs a combine kernel
- * merges.  These lists and an fp32 workspace for the parts (parts x 256 rows
- * x (head_dim + 1) x 4 bytes, e.g. 27 MB at 1024^2 with five references) are
- * one more cudaMalloc, freed by refcache_destroy.
+ * list of the step: when its (query tile, head) items do not fill the last
+ * round of the GPU's CTA pairs evenly, the items of that round are split by
+ * key range into 2-8 parts whose outputs a combine kernel merges.  This list
+ * and an fp32 workspace for the parts (parts x 256 rows x (head_dim + 1) x 4
+ * bytes, e.g. 27 MB at 1024^2 with five references) are one more cudaMalloc,
+ * freed by refcache_destroy.  Which step items are split depends on the whole
+ * batch and the device, so a step output's last bits may differ between
+ * batches (never by more than the rounding of a split).  The prefill is never
+ * split: refcache_build's outputs and cache bytes for a request depend only on
+ * that request's own inputs, whatever else is in the batch and on any GPU.
  */
 REFCACHE_API int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refcache_segments_t* seg,
                     void* dev_mem, size_t dev_bytes);
@@ -248,12 +252,19 @@ REFCACHE_API int full_attention(int batch, int num_heads, int head_dim, const in
  * GPU that loads the library until the process exits), so the call allocates
  * nothing: no cudaMalloc, no cudaFree, no allocating library routine.  The
  * caller still passes (and owns) q, k, v, o and lse.
- *   - The array holds REFCACHE_NOALLOC_MAX_TASKS work items; a request of n
- *     rows needs ceil(n / 128) of them.  Larger inputs are rejected with
+ *   - The array holds REFCACHE_NOALLOC_MAX_TASKS work items (512 KiB).  One
+ *     item covers up to 128 query rows of a request at head_dim 64 and up to
+ *     256 at head_dim 128, so a request of n rows needs ceil(n / 128) items at
+ *     head_dim 64 and ceil(n / 256) at head_dim 128: at most 16384 x 128 rows
+ *     per call at head_dim 64, 16384 x 256 at head_dim 128 (fewer when
+ *     requests end mid-item).  Larger inputs are rejected with
  *     REFCACHE_ERR_INVALID_ARG and a message naming the limit.
  *   - The first call on each device looks up the array's device address with
- *     that device current (a one-time set-up); make that first call before any
- *     stream capture.
+ *     that device current (a one-time set-up).
+ *   - Not capturable in a CUDA graph: each call copies its work list from a
+ *     host staging array (pageable memory) to the device array, which a stream
+ *     capture does not accept, and a replay would reread whatever the last
+ *     call left there.
  *   - Every call rewrites the whole work list it uses, so no state carries
  *     over, but all calls share the one array: calls whose kernels overlap on
  *     the GPU (different streams, or other threads) race.  Order them on one
@@ -268,6 +279,11 @@ REFCACHE_API int full_attention_noalloc(int batch, int num_heads, int head_dim, 
  * Synchronise `stream`, then read and clear the current device's error word
  * written by kernels whose bounded waits ran out.  Returns REFCACHE_OK,
  * REFCACHE_ERR_TIMEOUT or REFCACHE_ERR_CUDA.
+ * The word is one per device, not one per cache: every kernel of this library
+ * on the device (any cache, any stream, full_attention too) writes the same
+ * word, and the first refcache_status call that reads it clears it.  With
+ * several caches in flight on one device a timeout therefore says that some
+ * launch on the device gave up, not which cache's.
  */
 REFCACHE_API int refcache_status(void* stream);
 

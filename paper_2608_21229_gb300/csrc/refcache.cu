@@ -517,10 +517,10 @@ struct refcache {
   int n_step = 0;
   CopySeg* d_copy = nullptr;
   int n_copy = 0;
-  // per-item lists of the head-dim-128 kernel with split items, in a separate
-  // allocation: [build items | step items | build jobs | step jobs | part_o | part_lse]
+  // per-item list of the head-dim-128 step with split items, in a separate
+  // allocation: [step items | step jobs | part_o | part_lse]
   uint8_t* aux = nullptr;
-  ItemList build_items, step_items;
+  ItemList step_items;
   __nv_bfloat16* slots = nullptr;
   int64_t slot_elems = 0;
   // E4M3 cache (REFCACHE_CACHE_FP8): per layer [k8 | vt8 | scales] of
@@ -668,29 +668,25 @@ int check_ptrs(std::initializer_list<const void*> ps, int64_t rows, const char* 
   return REFCACHE_OK;
 }
 
-// Per-item lists (with the last round of items split) for the prefill and
-// the step of a head-dim-128 handle, in one allocation of their own (the
-// caller-sized cache memory is not touched).
-int plan_split_items(refcache* h, DeviceInfo* info, const std::vector<Task>& bt, const std::vector<Task>& st) {
+// Per-item list of the step of a head-dim-128 handle, with the last round of
+// items split, in one allocation of its own (the caller-sized cache memory is
+// not touched).  The prefill is never split: each of its items runs whole on
+// one CTA pair, so a request's prefill outputs depend on its own (N_ST, N_R)
+// only -- not on the other requests of the batch, nor on the device's SM count
+// -- and the cached block is reproduced bit for bit (Sec. 3.3).
+int plan_split_items(refcache* h, DeviceInfo* info, const std::vector<Task>& st) {
   int clusters = 0;
   int rc = tc2_clusters<false>(info, &clusters);
   if (rc) return rc;
-  int clusters_step = clusters;
-  if (h->f8 && h->rows_pad > 0 && (rc = tc2_clusters<true>(info, &clusters_step)) != 0) return rc;
-  std::vector<Task> bi, si;
-  std::vector<CombineJob> bj, sj;
-  int bparts = 0, sparts = 0;
-  plan_items(bt, h->H, clusters, &bi, &bj, &bparts);
-  plan_items(st, h->H, clusters_step, &si, &sj, &sparts);
-  const int parts = std::max(bparts, sparts);  // build and step calls are stream-ordered: one workspace
+  if (h->f8 && h->rows_pad > 0 && (rc = tc2_clusters<true>(info, &clusters)) != 0) return rc;
+  std::vector<Task> si;
+  std::vector<CombineJob> sj;
+  int parts = 0;
+  plan_items(st, h->H, clusters, &si, &sj, &parts);
   const int rows = task_rows(h->D);
   size_t off = 0;
-  const size_t o_bi = off;
-  off = align_up(off + bi.size() * sizeof(Task), 256);
   const size_t o_si = off;
   off = align_up(off + si.size() * sizeof(Task), 256);
-  const size_t o_bj = off;
-  off = align_up(off + bj.size() * sizeof(CombineJob), 256);
   const size_t o_sj = off;
   off = align_up(off + sj.size() * sizeof(CombineJob), 256);
   const size_t o_po = off;
@@ -700,25 +696,20 @@ int plan_split_items(refcache* h, DeviceInfo* info, const std::vector<Task>& bt,
   cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&h->aux), off);
   if (e != cudaSuccess) {
     h->aux = nullptr;
-    return fail(REFCACHE_ERR_OOM, "cudaMalloc(%zu) for the split work lists: %s", off, cudaGetErrorString(e));
+    return fail(REFCACHE_ERR_OOM, "cudaMalloc(%zu) for the split work list: %s", off, cudaGetErrorString(e));
   }
   auto put = [&](size_t o, const void* src, size_t n) -> cudaError_t {
     return n ? cudaMemcpy(h->aux + o, src, n, cudaMemcpyHostToDevice) : cudaSuccess;
   };
-  if ((e = put(o_bi, bi.data(), bi.size() * sizeof(Task))) != cudaSuccess ||
-      (e = put(o_si, si.data(), si.size() * sizeof(Task))) != cudaSuccess ||
-      (e = put(o_bj, bj.data(), bj.size() * sizeof(CombineJob))) != cudaSuccess ||
+  if ((e = put(o_si, si.data(), si.size() * sizeof(Task))) != cudaSuccess ||
       (e = put(o_sj, sj.data(), sj.size() * sizeof(CombineJob))) != cudaSuccess) {
     cudaFree(h->aux);
     h->aux = nullptr;
-    return cuda_fail(e, "cudaMemcpy(split work lists)");
+    return cuda_fail(e, "cudaMemcpy(split work list)");
   }
-  float* po = reinterpret_cast<float*>(h->aux + o_po);
-  float* pl = reinterpret_cast<float*>(h->aux + o_pl);
-  h->build_items = ItemList{reinterpret_cast<Task*>(h->aux + o_bi), static_cast<int>(bi.size()),
-                            reinterpret_cast<CombineJob*>(h->aux + o_bj), static_cast<int>(bj.size()), po, pl};
   h->step_items = ItemList{reinterpret_cast<Task*>(h->aux + o_si), static_cast<int>(si.size()),
-                           reinterpret_cast<CombineJob*>(h->aux + o_sj), static_cast<int>(sj.size()), po, pl};
+                           reinterpret_cast<CombineJob*>(h->aux + o_sj), static_cast<int>(sj.size()),
+                           reinterpret_cast<float*>(h->aux + o_po), reinterpret_cast<float*>(h->aux + o_pl)};
   return REFCACHE_OK;
 }
 
@@ -801,7 +792,7 @@ int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refca
     delete h;
     return cuda_fail(e, "cudaMemcpy(work tables)");
   }
-  if (h->D == 128 && (rc = plan_split_items(h, info, bt, st)) != 0) {
+  if (h->D == 128 && (rc = plan_split_items(h, info, st)) != 0) {
     if (h->owns) cudaFree(h->mem);
     delete h;
     return rc;
@@ -855,9 +846,9 @@ int refcache_call_launches(refcache_t* h, int call) {
   const int n_tasks = call == 0 ? h->n_build : h->n_step;
   const int cache_write = call == 0 && (h->n_copy > 0 || h->n_qtiles > 0) ? 1 : 0;
   if (n_tasks == 0) return cache_write;
-  const ItemList& il = call == 0 ? h->build_items : h->step_items;
   const bool tc = g_kernel.load() == REFCACHE_KERNEL_TCGEN05;
-  return cache_write + 1 + (tc && il.items && il.n_jobs > 0 ? 1 : 0);
+  const bool combine = call == 1 && tc && h->step_items.items && h->step_items.n_jobs > 0;
+  return cache_write + 1 + (combine ? 1 : 0);
 }
 
 int refcache_layer_built(refcache_t* h, int layer) {
@@ -898,8 +889,8 @@ int refcache_build(refcache_t* h, int layer, const void* q_static, const void* k
     cj.rows = h->cache_rows;
   }
   Operands op{q_static, h->static_rows, k_static, v_static, h->static_rows, nullptr, nullptr, 0, o_static, lse_static};
-  rc = run_attention(h->d_build, h->n_build, h->H, h->D, op, softmax_scale, info, s,
-                     h->build_items.items ? &h->build_items : nullptr, nullptr, h->n_copy > 0 ? &cj : nullptr);
+  rc = run_attention(h->d_build, h->n_build, h->H, h->D, op, softmax_scale, info, s, nullptr, nullptr,
+                     h->n_copy > 0 ? &cj : nullptr);
   if (rc) return rc;
   h->built[layer] = 1;
   return REFCACHE_OK;

@@ -74,8 +74,10 @@ def test_edit1024_5ref_sampled(kernel):
     pu.sampled_compare(run, seed=5)
 
 
-@pytest.mark.parametrize("refs", [1, 10])
+@pytest.mark.parametrize("refs", [1, 2, 8, 10])
 def test_sweep_sampled(refs):
+    """The reference-scaling sweep at 1024^2 (5 references is the headline
+    test above): prefill and step sampled against the oracle."""
     w = [x for x in workloads.SWEEP_1024 if x.requests[0].n_r == refs * 4096][0]
     run = pu.GpuRun(w, kernel="tcgen05")
     pu.sampled_compare(run, seed=refs, per_request=16)
@@ -170,6 +172,32 @@ def test_full_attention_matches_oracle(kernel, w):
     pu.check_close(go, ref_o, gl, ref_l, "full")
 
 
+def test_full_attention_sampled_edit1024_5ref():
+    """The recompute baseline at the size the benchmark times it: [LT; X; R] of
+    the 1024^2, five-reference edit (25,088 rows, 24 heads), every row over
+    every key (C_full in App. C).  Rows at the 256-row task edges, the ragged
+    tail and random rows, against the oracle one by one."""
+    rcb.set_kernel("tcgen05")
+    r = workloads.EDIT_1024_5REF.requests[0]
+    n = r.n_lt + r.n_x + r.n_r
+    H, D = 24, 128
+    q, k, v = (workloads.randn_bf16((n, H, D), 2, f"full_{t}") for t in "qkv")
+    o = torch.full((n, H, D), float("nan"), dtype=torch.bfloat16, device="cuda")
+    lse = torch.full((n, H), float("nan"), dtype=torch.float32, device="cuda")
+    rcb.full_attention([0, n], q.cuda(), k.cuda(), v.cuda(), o, lse)
+    torch.cuda.synchronize()
+    assert rcb.status() == rcb.OK
+    rng = np.random.default_rng(25088)
+    rows = set(int(x) for x in pu.sample_rows(n, rng, 40))
+    rows |= {256 * t + e for t in (1, 17, 50, 97) for e in (-1, 0)} | {n - 256, n - 255}
+    rows = np.array(sorted(x for x in rows if 0 <= x < n), np.int64)
+    pairs = np.stack([rows, rng.integers(0, H, rows.size)], 1).astype(np.int32)
+    ref_o, ref_l = oracle.full(pu.bits(q), pu.bits(k), pu.bits(v), 1 / math.sqrt(D), pairs)
+    go = pu.f64(o)[pairs[:, 0], pairs[:, 1]]
+    gl = pu.f64(lse)[pairs[:, 0], pairs[:, 1]]
+    pu.check_close(go, ref_o, gl, ref_l, "full 1024^2 x 5 refs")
+
+
 def test_kernels_agree_closely():
     """The two kernels compute the same function (different rounding order)."""
     w = workloads.EDIT_512_2REF
@@ -220,11 +248,13 @@ def test_cfg_edit1024_5ref_sampled():
 
 @pytest.mark.parametrize("w", [workloads.CFG_SMALL, workloads.CFG_1024_5REF], ids=lambda w: w.name)
 def test_cfg_pair_equals_branches_run_alone(w):
-    """Both branches in one launch give what each branch gives alone: the
-    caches bit for bit, most outputs bit for bit, and every output within a
-    tenth of the parity bar (a launch splits the items of its last round by
-    key range, and which items those are depends on the launch's item count;
-    each part rounds P against its own running maximum)."""
+    """Both branches in one launch give what each branch gives alone.  The
+    prefill (outputs, LSE and cache) bit for bit: its items are never split,
+    so a request's static block does not depend on what else is in the batch
+    (Sec. 3.3).  The step: most outputs bit for bit and every output within a
+    tenth of the parity bar (a step launch splits the items of its last round
+    by key range, and which items those are depends on the launch's item
+    count; each part rounds P against its own running maximum)."""
     pair = pu.GpuRun(w, kernel="tcgen05")
     for b, r in enumerate(w.requests):
         single = workloads.Workload(f"{w.name}_branch{b}", w.num_heads, w.head_dim, (r,), w.seed)
@@ -232,11 +262,13 @@ def test_cfg_pair_equals_branches_run_alone(w):
         static = tuple(t[s0:s0 + r.n_static] for t in pair.static)
         live = tuple(t[l0:l0 + r.n_live] for t in pair.live)
         alone = pu.GpuRun(single, kernel="tcgen05", static=static, live=live)
-        for got, ref in ((pair.o_live[l0:l0 + r.n_live], alone.o_live),
-                         (pair.o_static[s0:s0 + r.n_static], alone.o_static)):
-            g, a = pu.f64(got), pu.f64(ref)
-            assert np.max(np.abs(g - a)) <= pu.MAX_ABS / 10
-            assert np.mean(pu.bits(got) == pu.bits(ref)) > 0.5
+        assert np.array_equal(pu.bits(pair.o_static[s0:s0 + r.n_static]), pu.bits(alone.o_static))
+        ls_pair = pair.lse_static[s0:s0 + r.n_static].cpu().view(torch.int32)
+        assert torch.equal(ls_pair, alone.lse_static.cpu().view(torch.int32))
+        got, ref = pair.o_live[l0:l0 + r.n_live], alone.o_live
+        g, a = pu.f64(got), pu.f64(ref)
+        assert np.max(np.abs(g - a)) <= pu.MAX_ABS / 10
+        assert np.mean(pu.bits(got) == pu.bits(ref)) > 0.5
         c0 = pu.cache_offsets(w, "beyond")[b]
         assert np.array_equal(pu.bits(alone.k_cache), pu.bits(pair.k_cache[c0:c0 + r.n_r]))
         assert np.array_equal(pu.bits(alone.v_cache), pu.bits(pair.v_cache[c0:c0 + r.n_r]))
@@ -244,9 +276,9 @@ def test_cfg_pair_equals_branches_run_alone(w):
 
 # ---------------------------------------------------------------- split items (last round of the persistent grid)
 def test_split_tail_items_sampled():
-    """The last round of items of a launch is split by key range into parts
-    merged by a combine kernel; on the headline case those are items of the
-    last heads (head-major order), for both the prefill and the step."""
+    """The last round of items of a step launch is split by key range into
+    parts merged by a combine kernel; on the headline case those are items of
+    the last heads (head-major order)."""
     run = pu.GpuRun(workloads.EDIT_1024_5REF, kernel="tcgen05")
     pu.sampled_compare(run, seed=21, per_request=64, heads=[21, 22, 23])
 
@@ -258,14 +290,15 @@ def test_split_tail_items_cfg_pair_sampled():
 
 def test_call_launch_counts():
     """Kernels per call: attention (+ cache copy for the build) (+ combine when
-    the device's plan split the last round; the headline step's 432 items do
-    not fill 76 CTA pairs evenly, so it is split on a GB300)."""
+    the device's plan split the step's last round; the headline step's 432
+    items do not fill 76 CTA pairs evenly, so it is split on a GB300; the
+    prefill is never split)."""
     w = workloads.EDIT_1024_5REF
     seg = rcb.Segments.from_workload(w)
     cache = rcb.RefCache(seg, num_layers=1, mask_mode="beyond")
     rcb.set_kernel("tcgen05")
     assert cache.launches("step") in (1, 2)
-    assert cache.launches("build") == cache.launches("step") + 1
+    assert cache.launches("build") == 2
     rcb.set_kernel("mma_sync")
     assert cache.launches("step") == 1 and cache.launches("build") == 2
     rcb.set_kernel("tcgen05")
