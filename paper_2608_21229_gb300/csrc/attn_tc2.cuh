@@ -125,7 +125,12 @@ struct SmemT {
                        kNumBars = kScaleEmpty + kScaleSlots;
   static constexpr uint32_t kTmemHolder = kBars + 8 * kNumBars;
   static constexpr uint32_t kAbort = kTmemHolder + 4;
-  static constexpr uint32_t kUsed = kAbort + 4;
+  // load record of each CTA of the pair (leader's copy read at teardown):
+  // per CTA [loads per stage (kStages) | own bytes of the last load per stage
+  // (kStages) | loads per Q buffer (2)]
+  static constexpr uint32_t kRecWords = 2 * kStages + 2;
+  static constexpr uint32_t kLoadRec = kAbort + 4;
+  static constexpr uint32_t kUsed = kLoadRec + 2 * kRecWords * 4;
   static constexpr uint32_t kMaxDynamic = 232448;
   static constexpr uint32_t kDynamic = kUsed + 1024 < kMaxDynamic ? kUsed + 1024 : kMaxDynamic;
   static_assert(kUsed <= kMaxDynamic, "shared-memory layout too large");
@@ -244,9 +249,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
     // This CTA's halves of the stages of every group, in group order, and an
     // item's Q rows just before its first stage.
     if (lane == 0) {
-      int armed_phase[kStages];
-      for (int s = 0; s < kStages; ++s) armed_phase[s] = -1;
-      int q_armed[2] = {-1, -1};
+      // loads this CTA issued per stage and per Q buffer, and its bytes of the
+      // last load of each stage; the leader arms every phase for both CTAs'
+      // bytes right before it issues its own half
+      int n_stage[kStages];
+      uint32_t own_bytes[kStages];
+      for (int s = 0; s < kStages; ++s) {
+        n_stage[s] = 0;
+        own_bytes[s] = 0;
+      }
+      int n_q[2] = {0, 0};
       int scale_armed[tc2::kScaleSlots];
       for (int s = 0; s < tc2::kScaleSlots; ++s) scale_armed[s] = -1;
       bool skip_next = leader && args.dbg_skip_first_load != 0;
@@ -280,10 +292,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
         if (skip_next) {  // fault injection: the leader never arms or loads this stage
           skip_next = false;
         } else {
-          if (leader) {
-            mbar_arrive_expect_tx(bar(L::kStageFull + slot), bytes);
-            armed_phase[slot] = static_cast<int>(group_parity(g));
-          }
+          if (leader) mbar_arrive_expect_tx(bar(L::kStageFull + slot), bytes);
+          ++n_stage[slot];
+          own_bytes[slot] = bytes / 2;
           if (k8) {  // E4M3 keys [64 r, 64 r + 64): one box of 64 rows x 128 bytes
             tma_load_2d_pair(dst, &tm_kb, full, head * D, ks.row + 64 * static_cast<int>(rank));
           } else if (kj >= 0) {  // keys [64 r, 64 r + 64) of the tile, both head-dim boxes
@@ -309,10 +320,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
           const int b = qi & 1;
           const uint32_t n = static_cast<uint32_t>(qi >> 1);
           if (!wait_one(bar(L::kQEmpty + b), (n & 1u) ^ 1u, ctl, 1)) goto producer_done;
-          if (leader) {
-            mbar_arrive_expect_tx(bar(L::kQFull + b), 2 * kQTile);
-            q_armed[b] = static_cast<int>(n);
-          }
+          if (leader) mbar_arrive_expect_tx(bar(L::kQFull + b), 2 * kQTile);
+          ++n_q[b];
           const uint32_t qfull = lbar(L::kQFull + b);
           for (int ch = 0; ch < 2; ++ch)
             tma_load_2d_pair(base + L::kQ + b * kQTile + ch * kBoxBytes, &tm_q, qfull, head * D + ch * 64,
@@ -325,15 +334,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
         ++qi;
       }
     producer_done:
-      // the leader's full barriers count both CTAs' bytes: once they complete,
-      // every load of the pair has landed
-      for (int s = 0; s < kStages; ++s)
-        if (armed_phase[s] >= 0)
-          drain_one(bar(L::kStageFull + s), static_cast<uint32_t>(armed_phase[s]), args.timeout_ns);
-      for (int b = 0; b < 2; ++b)
-        if (q_armed[b] >= 0) drain_one(bar(L::kQFull + b), static_cast<uint32_t>(q_armed[b]) & 1u, args.timeout_ns);
+      // the scale ring's barriers are this CTA's own
       for (int s = 0; s < tc2::kScaleSlots; ++s)
         if (scale_armed[s] >= 0) drain_one(bar(L::kScaleFull + s), static_cast<uint32_t>(scale_armed[s]), args.timeout_ns);
+      // stage and Q loads of both CTAs complete on the leader's barriers: record
+      // this CTA's loads in the leader's shared memory, where the leader
+      // settles and drains them after the teardown's first cluster barrier
+      const uint32_t rec = mapa_shared(base + L::kLoadRec + rank * (L::kRecWords * 4u), 0);
+      for (int s = 0; s < kStages; ++s) {
+        st_cluster_u32(rec + 4u * s, static_cast<uint32_t>(n_stage[s]));
+        st_cluster_u32(rec + 4u * (kStages + s), own_bytes[s]);
+      }
+      st_cluster_u32(rec + 4u * (2 * kStages), static_cast<uint32_t>(n_q[0]));
+      st_cluster_u32(rec + 4u * (2 * kStages + 1), static_cast<uint32_t>(n_q[1]));
     }
     __syncwarp();
   } else if (warp == Cfg::kMmaWarp) {
@@ -850,11 +863,40 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
 
   tc_fence_before();
   __syncthreads();
-  cluster_sync();  // the pair's MMAs and TMEM reads are over in both CTAs
+  // the pair's MMAs and TMEM reads are over in both CTAs, and both producers'
+  // load records are in the leader's shared memory
+  cluster_sync();
   if (warp == Cfg::kMmaWarp) {
     tc_fence_after();
     tmem_dealloc_pair(tmem, kTmemCols);
   }
+  if (leader && warp == Cfg::kProducerWarp && lane == 0) {
+    // Every stage and Q load of either CTA must land before that CTA exits.
+    // The leader arms a phase for both halves before it issues its own, and
+    // each CTA issues its half after the same wait; after an abort the two can
+    // differ by one phase.  A phase the follower loaded but the leader never
+    // armed is armed now for the follower's bytes; a phase the leader armed
+    // whose follower half was never issued has those bytes counted as
+    // arrived.  Then the last phase of every barrier is drained (bounded).
+    const volatile uint32_t* rec = reinterpret_cast<const volatile uint32_t*>(base_ptr + L::kLoadRec);
+    const volatile uint32_t* peer = rec + L::kRecWords;
+    auto settle = [&](uint32_t b, int mine, int theirs, uint32_t mine_bytes, uint32_t their_bytes) {
+      if (theirs == mine + 1) {
+        mbar_arrive_expect_tx(b, their_bytes);
+        mine = theirs;
+      } else if (mine == theirs + 1 && mine_bytes > 0) {
+        mbar_complete_tx(b, mine_bytes);
+      }
+      if (mine > 0) drain_one(b, static_cast<uint32_t>(mine - 1) & 1u, args.timeout_ns);
+    };
+    for (int s = 0; s < kStages; ++s)
+      settle(bar(L::kStageFull + s), static_cast<int>(rec[s]), static_cast<int>(peer[s]), rec[kStages + s],
+             peer[kStages + s]);
+    for (int b = 0; b < 2; ++b)
+      settle(bar(L::kQFull + b), static_cast<int>(rec[2 * kStages + b]), static_cast<int>(peer[2 * kStages + b]),
+             kQTile, kQTile);
+  }
+  // the follower leaves only once the leader has seen every load of the pair land
   cluster_sync();
 }
 
