@@ -164,6 +164,17 @@ def dequantized_cache(k8, vt8, scales, seg_off, cached_rows_per_request):
     return np.concatenate(ks), np.concatenate(vs)
 
 
+def cached_v_scales(scales, seg_off, cached_rows_per_request):
+    """s_V of the tile each cached row belongs to: float64 [sum n_b, H]."""
+    out = []
+    for b, n in enumerate(cached_rows_per_request):
+        rows = np.arange(seg_off[b], seg_off[b] + n)
+        out.append(scales[rows // TILE, :, 1].astype(np.float64))
+    if not out:
+        return np.zeros((0, scales.shape[1]))
+    return np.concatenate(out)
+
+
 def quantize_queries(q_bits):
     """Per (row, head) quantisation of the step's queries: (codes [n, H, d], s [n, H])."""
     q = bf16_to_f32(q_bits)
@@ -176,7 +187,7 @@ def quantize_queries(q_bits):
     return codes, s
 
 
-def step_fp8(q_l, k_l, v_l, k_cache_deq, v_cache_deq, scale, pairs, bound=False):
+def step_fp8(q_l, k_l, v_l, k_cache_deq, v_cache_deq, scale, pairs, bound=False, v_scale=None):
     """One request's step over the quantised cache, for the (live row, head)
     pairs given: returns (out [P, d], lse [P]) in fp64.
 
@@ -187,16 +198,31 @@ def step_fp8(q_l, k_l, v_l, k_cache_deq, v_cache_deq, scale, pairs, bound=False)
     App. C's step for live rows, with the cache holding R or [ST; R]).
 
     With ``bound``, also returns [P, d] worst-case bounds of what rounding
-    the softmax weights can add to each output (the CUDA path rounds the
-    weights of cached keys to E4M3 and those of live keys to bf16, and its
-    output to bf16).  With w_k = exp(s_k - max) and l = sum w_k: a weight
-    rounded to E4M3 is off by at most 2^-4 w_k in the normal range and by
-    half the subnormal step, 2^-10, below it (taken as 2^-9, so that the
-    kernel's per-tile shift of the weights by at most a factor two below the
-    first tile's V scale is covered); a bf16 weight by 2^-9 w_k; the bf16
-    output by 2^-8 |o| (half an ulp is 2^-9 relative, doubled for margin):
-        bound_c = (sum_cache (2^-4 w_k + 2^-9) |v_kc| + sum_live 2^-9 w_k |v_kc|) / l + 2^-8 |o_c|
+    the softmax weights adds to each output under the variant's weight rule;
+    ``v_scale`` [n_cached, H] then gives s_V of each cached row's tile
+    (``cached_v_scales``).  The rule: with u = score x log2(e), s_ref the V
+    scale of one cached tile of the request, delta_t = log2(s_V,t / s_ref) and
+    m a running maximum of u (live keys) and u + delta_t (cached keys), a
+    cached key's weight exp2(u + delta_t - m) is stored as E4M3 and multiplies
+    its V code, a live key's weight exp2(u - m) / s_ref is stored as bf16 and
+    multiplies its V, the sum is scaled by s_ref and divided by
+    l = sum exp2(u - m); the output is rounded to bf16.  Then, with
+    w_k = exp(s_k - max) and den = sum w_k:
+      * an E4M3 weight is off by at most 2^-4 of itself (normal range) plus
+        half the subnormal step, 2^-10.  The relative part maps to
+        2^-4 w_k |v_kc| / den.  The absolute part maps to
+        2^-10 (s_ref / s_V,t) 2^(m - M) |v_kc| / den, M the largest u; m - M
+        is at most max_t delta_t, so the factor is at most s_V,max / s_V,t
+        (s_ref cancels; s_V,max = the largest V scale of the request's
+        cached tiles);
+      * a bf16 weight is off by at most 2^-9 of itself: 2^-9 w_k |v_kc| / den;
+      * the bf16 output by half an ulp, 2^-9 |o_c|, doubled for margin:
+        bound_c = (sum_cache (2^-4 w_k + 2^-10 s_V,max / s_V,t(k)) |v_kc|
+                   + sum_live 2^-9 w_k |v_kc|) / den + 2^-8 |o_c|
+    (a tile with s_V = 0 holds V = 0 and adds nothing).
     """
+    if bound and v_scale is None:
+        raise ValueError("the weight-rounding bound needs the cached rows' V tile scales (v_scale)")
     qf = bf16_to_f32(q_l).astype(np.float64)
     kf = bf16_to_f32(k_l).astype(np.float64)
     vf = bf16_to_f32(v_l).astype(np.float64)
@@ -223,7 +249,9 @@ def step_fp8(q_l, k_l, v_l, k_cache_deq, v_cache_deq, scale, pairs, bound=False)
         lse[p] = m + np.log(den)
         if bound:
             av = np.abs(vals)
-            bnd[p] = ((2.0 ** -4 * w[n_live:] + 2.0 ** -9) @ av[n_live:]
+            sv = v_scale[:, h]
+            ratio = np.where(sv > 0, (sv.max() if sv.size else 0.0) / np.where(sv > 0, sv, 1.0), 0.0)
+            bnd[p] = ((2.0 ** -4 * w[n_live:] + 2.0 ** -10 * ratio) @ av[n_live:]
                       + 2.0 ** -9 * w[:n_live] @ av[:n_live]) / den + 2.0 ** -8 * np.abs(out[p])
     if bound:
         return out, lse, bnd

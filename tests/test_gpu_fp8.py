@@ -99,6 +99,7 @@ def check_step(run, heads, rows_per_request=None, seed=0, statistical=True):
     scale = 1.0 / math.sqrt(w.head_dim)
     k8, vt8, sc, off, lens = check_cache(run, heads)
     kd, vd = ofp8.dequantized_cache(k8, vt8, sc, off, lens)
+    vsc = ofp8.cached_v_scales(sc, off, lens)
     cum = np.concatenate([[0], np.cumsum(lens)])
     o_l, l_l = pu.f64(run.o_live), pu.f64(run.lse_live)
     rng = np.random.default_rng(seed)
@@ -117,7 +118,7 @@ def check_step(run, heads, rows_per_request=None, seed=0, statistical=True):
         pairs = np.stack([rows, hj], 1)
         q, k, v = (pu.bits(t)[l0:l0 + r.n_live][:, heads] for t in run.live)
         ref_o, ref_l, bnd = ofp8.step_fp8(q, k, v, kd[cum[b]:cum[b + 1]], vd[cum[b]:cum[b + 1]], scale, pairs,
-                                          bound=True)
+                                          bound=True, v_scale=vsc[cum[b]:cum[b + 1]])
         hs = np.asarray(heads)[hj]
         g_o = o_l[l0 + rows, hs]
         assert np.isfinite(g_o).all(), f"step req {b}: non-finite output"

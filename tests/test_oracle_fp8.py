@@ -187,12 +187,12 @@ def _fp8_case(seed, n_live, n_cached, H=2, d=128):
     q_l, k_l, v_l, k_c, v_c = bits(n_live), bits(n_live), bits(n_live), bits(n_cached), bits(n_cached)
     k8, vt8, sc, off = fp8.build_fp8_cache(k_c, v_c, [n_cached])
     kd, vd = fp8.dequantized_cache(k8, vt8, sc, off, [n_cached])
-    return q_l, k_l, v_l, k_c, v_c, kd, vd
+    return q_l, k_l, v_l, k_c, v_c, kd, vd, fp8.cached_v_scales(sc, off, [n_cached])
 
 
 def test_fp8_step_close_to_exact_step(oracle_mod):
     """The approximation itself: N(0,1) inputs, error of the quantised step."""
-    q_l, k_l, v_l, k_c, v_c, kd, vd = _fp8_case(17, 96, 700)
+    q_l, k_l, v_l, k_c, v_c, kd, vd, _ = _fp8_case(17, 96, 700)
     pairs = np.array([(i, h) for i in range(0, 96, 5) for h in range(2)])
     scale = 1.0 / np.sqrt(128)
     o8, l8 = fp8.step_fp8(q_l, k_l, v_l, kd, vd, scale, pairs)
@@ -202,22 +202,34 @@ def test_fp8_step_close_to_exact_step(oracle_mod):
     assert np.abs(l8 - l).max() < 2e-2
 
 
-def _weights_rounded(q_l, k_l, v_l, kd, vd, scale, pairs):
-    """The CUDA path's extra rounding, simulated: softmax weights of live keys
-    to bf16 and of cached keys to E4M3 (relative to the row maximum), the
-    normaliser from the unrounded weights."""
+def _weights_rounded(q_l, k_l, v_l, kd, vd, vsc, scale, pairs, lag=0.0):
+    """The CUDA path's extra rounding, simulated by the variant's weight rule
+    (reading R12): scores in log2 units u, s_ref = the first cached tile's V
+    scale, delta = log2(s_V,t / s_ref) per cached tile, m = max over the live
+    u and the cached u + delta, lowered by ``lag`` (the running maximum may
+    trail the true one by up to 8 before a rescale); cached weights
+    exp2(u + delta - m) rounded to E4M3 times the V codes, live weights
+    exp2(u - m) / s_ref rounded to bf16 times V, the sum times s_ref over the
+    unrounded l = sum exp2(u - m)."""
     qf = fp8.bf16_to_f32(q_l).astype(np.float64)
     kf = fp8.bf16_to_f32(k_l).astype(np.float64)
     vf = fp8.bf16_to_f32(v_l).astype(np.float64)
     out = np.zeros((len(pairs), qf.shape[2]))
+    n_live = kf.shape[0]
     for p, (i, h) in enumerate(pairs):
         codes, sq = fp8.quantize_block(fp8.bf16_to_f32(q_l[i, h]))
-        s = np.concatenate([kf[:, h] @ qf[i, h], kd[:, h] @ (float(sq) * fp8.e4m3_decode(codes))]) * scale
-        w = np.exp(s - s.max())
-        n_live = kf.shape[0]
-        w_live = torch.from_numpy(w[:n_live].astype(np.float32)).to(torch.bfloat16).to(torch.float64).numpy()
-        w_cache = fp8.e4m3_decode(fp8.e4m3_encode(w[n_live:].astype(np.float32)))
-        out[p] = (w_live @ vf[:, h] + w_cache @ vd[:, h]) / w.sum()
+        u = np.concatenate([kf[:, h] @ qf[i, h], kd[:, h] @ (float(sq) * fp8.e4m3_decode(codes))]) * scale
+        u = u * np.log2(np.e)
+        sv = vsc[:, h]
+        s_ref = sv[0] if sv.size and sv[0] > 0 else 1.0
+        delta = np.where(sv > 0, np.log2(np.where(sv > 0, sv, 1.0) / s_ref), 0.0)
+        m = max(u[:n_live].max(initial=-np.inf), (u[n_live:] + delta).max(initial=-np.inf)) - lag
+        l = np.exp2(u - m).sum()
+        w_live = np.exp2(u[:n_live] - m) / s_ref
+        w_live = torch.from_numpy(w_live.astype(np.float32)).to(torch.bfloat16).to(torch.float64).numpy()
+        w_cache = fp8.e4m3_decode(fp8.e4m3_encode(np.exp2(u[n_live:] + delta - m).astype(np.float32)))
+        codes_v = np.where(sv[:, None] > 0, vd[:, h] / np.where(sv > 0, sv, 1.0)[:, None], 0.0)
+        out[p] = s_ref * (w_live @ vf[:, h] + w_cache @ codes_v) / l
     return out
 
 
@@ -226,10 +238,10 @@ def test_weight_rounding_bound_on_few_keys():
     worst-case bound must still hold, and be reached within a factor of ten."""
     worst = 0.0
     for seed in range(6):
-        q_l, k_l, v_l, k_c, v_c, kd, vd = _fp8_case(40 + seed, 2, 5)
+        q_l, k_l, v_l, k_c, v_c, kd, vd, vsc = _fp8_case(40 + seed, 2, 5)
         pairs = np.array([(i, h) for i in range(2) for h in range(2)])
-        o8, _, bnd = fp8.step_fp8(q_l, k_l, v_l, kd, vd, 1.0 / np.sqrt(128), pairs, bound=True)
-        sim = _weights_rounded(q_l, k_l, v_l, kd, vd, 1.0 / np.sqrt(128), pairs)
+        o8, _, bnd = fp8.step_fp8(q_l, k_l, v_l, kd, vd, 1.0 / np.sqrt(128), pairs, bound=True, v_scale=vsc)
+        sim = _weights_rounded(q_l, k_l, v_l, kd, vd, vsc, 1.0 / np.sqrt(128), pairs)
         err = np.abs(sim - o8)
         assert np.all(err <= bnd)
         worst = max(worst, float((err / bnd).max()))
@@ -238,14 +250,41 @@ def test_weight_rounding_bound_on_few_keys():
 
 @pytest.mark.parametrize("n_live,n_cached", [(64, 400), (96, 1024), (300, 2048)])
 def test_gpu_fp8_tolerance_covers_weight_rounding(n_live, n_cached):
-    q_l, k_l, v_l, k_c, v_c, kd, vd = _fp8_case(18 + n_cached, n_live, n_cached)
+    q_l, k_l, v_l, k_c, v_c, kd, vd, vsc = _fp8_case(18 + n_cached, n_live, n_cached)
     pairs = np.array([(i, h) for i in range(0, n_live, 3) for h in range(2)])
     scale = 1.0 / np.sqrt(128)
-    o8, _, bnd = fp8.step_fp8(q_l, k_l, v_l, kd, vd, scale, pairs, bound=True)
-    sim = _weights_rounded(q_l, k_l, v_l, kd, vd, scale, pairs)
+    o8, _, bnd = fp8.step_fp8(q_l, k_l, v_l, kd, vd, scale, pairs, bound=True, v_scale=vsc)
+    sim = _weights_rounded(q_l, k_l, v_l, kd, vd, vsc, scale, pairs)
     err = np.abs(sim - o8)
     assert np.all(err <= bnd)  # the analytic worst case holds
+    lagged = _weights_rounded(q_l, k_l, v_l, kd, vd, vsc, scale, pairs, lag=8.0)
+    assert np.all(np.abs(lagged - o8) <= bnd)  # and with the running maximum trailing by 2^8
     # the rounding error must sit well inside the tolerance (margin for fp32
     # arithmetic, the bf16 output and rows the sample did not draw)
     assert err.max() < FP8_MAX_ABS / 2
     assert err.mean() < FP8_MEAN_ABS / 2
+
+
+@pytest.mark.parametrize("first_tile_gain", [1.0 / 16, 16.0])
+def test_weight_rounding_bound_with_uneven_v_scales(first_tile_gain):
+    """V tiles whose scales differ by 16x (the first tile, whose scale is
+    s_ref, the smallest or the largest): the bound's absolute term, which
+    scales with s_V,max / s_V,t, must still cover the variant's rounding, with
+    the running maximum exact or trailing by 2^8."""
+    rng = np.random.default_rng(77 if first_tile_gain < 1 else 78)
+    H, d, n_live, n_cached = 2, 128, 24, 3 * fp8.TILE
+    bits = lambda x: workloads.bf16_bits(torch.from_numpy(x.astype(np.float32)).to(torch.bfloat16))  # noqa: E731
+    q_l, k_l, v_l = (bits(rng.standard_normal((n_live, H, d))) for _ in range(3))
+    k_c = bits(2.0 * rng.standard_normal((n_cached, H, d)))  # peaked softmax: many subnormal weights
+    v = rng.standard_normal((n_cached, H, d))
+    v[:fp8.TILE] *= first_tile_gain
+    v_c = bits(v)
+    k8, vt8, sc, off = fp8.build_fp8_cache(k_c, v_c, [n_cached])
+    kd, vd = fp8.dequantized_cache(k8, vt8, sc, off, [n_cached])
+    vsc = fp8.cached_v_scales(sc, off, [n_cached])
+    pairs = np.array([(i, h) for i in range(0, n_live, 2) for h in range(H)])
+    scale = 1.0 / np.sqrt(d)
+    o8, _, bnd = fp8.step_fp8(q_l, k_l, v_l, kd, vd, scale, pairs, bound=True, v_scale=vsc)
+    for lag in (0.0, 8.0):
+        sim = _weights_rounded(q_l, k_l, v_l, kd, vd, vsc, scale, pairs, lag=lag)
+        assert np.all(np.abs(sim - o8) <= bnd), f"lag {lag}"
