@@ -342,8 +342,9 @@ def run_ours(args, ws, rank, local):
         },
         "roofline": {
             "kernel": ("attn_mma_kernel (mma.sync)" if args.kernel == "mma_sync" else
-                       "attn_tc2_kernel (tcgen05, CTA pairs)" if D == 128 else "attn_tc_kernel<64> (tcgen05)")
-                      + " in step_attention",
+                       "attn_tc2_kernel (tcgen05, CTA pairs, 128-key tiles)" if D == 128 and args.kernel == "tcgen05_k128"
+                       else "attn_tc2_kernel (tcgen05, CTA pairs, 192-key tiles)" if D == 128
+                       else "attn_tc_kernel<64> (tcgen05)") + " in step_attention",
             "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
             "frac": achieved / peak,
             "peak_kind": (f"bf16 dense, {pk['source']} burst (the timed region runs near the maximum SM clock)"
@@ -836,7 +837,7 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="edit1024_5ref")
-    ap.add_argument("--kernel", choices=["tcgen05", "mma_sync"], default="tcgen05")
+    ap.add_argument("--kernel", choices=["tcgen05", "tcgen05_k128", "mma_sync"], default="tcgen05")
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--ref-pairs", type=int, default=192, help="oracle (row, head) outputs per reference step")
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -113,9 +113,13 @@ extern "C" {
 #define REFCACHE_CACHE_FP8 0x100
 
 /* Kernel selection (refcache_set_kernel): the tcgen05/TMEM/TMA kernel is the
- * default; the mma.sync kernel is the recompiled legacy-tensor-core baseline. */
+ * default (at head_dim 128 on CTA pairs with 192-key tiles for the bf16
+ * cache); the mma.sync kernel is the recompiled legacy-tensor-core baseline;
+ * TCGEN05_K128 is the same tcgen05 pair kernel with 128-key tiles, kept as a
+ * comparison point (head_dim 64 and the E4M3 cache always use 128-key tiles). */
 #define REFCACHE_KERNEL_TCGEN05 0
 #define REFCACHE_KERNEL_MMA_SYNC 1
+#define REFCACHE_KERNEL_TCGEN05_K128 2
 
 /*
  * Segment table of a batch of requests (Eq. 1 layout, Sec. 3.3 order).

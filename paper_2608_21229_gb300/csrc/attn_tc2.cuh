@@ -88,40 +88,57 @@ namespace rc {
 namespace tc2 {
 using tc::Ctl;
 constexpr int kD = 128;
-constexpr int kStages = 4;                  // ring stages (pair_done has as many barriers)
-constexpr uint32_t kKHalf = 64 * 128 * 2;   // 16 KB: this CTA's 64 keys x 128 d of a K tile
-constexpr uint32_t kVHalf = 128 * 64 * 2;   // 16 KB: 128 keys x this CTA's 64 d of a V tile
-constexpr uint32_t kStage = kKHalf + kVHalf;
 constexpr uint32_t kQTile = 128 * 128 * 2;
-constexpr uint32_t kKBox = 64 * 128;        // one K box: 64 rows x 128 bytes
 // Warp roles: softmax warps first (4, or 8 in the E4M3 kernel, two per SM
 // sub-partition), then the producer, the MMA warp and the gate warp.
-template <bool kF8>
+//
+// kBN = keys per tile: 128, or 192 for the bf16 cache.  With 192-key tiles P
+// is written over the first half of its own S buffer, so that tensor memory
+// holds S_0 [0, 192), S_1 [192, 384) and O [384, 512); an MMA group is then
+// 12 P.V MMAs and 8 S MMAs of N = 192 (1536 tensor cycles per handshake
+// instead of 1024), and since the S MMAs that reuse a buffer overwrite the P
+// that the group's P.V MMAs read, a group issues all its P.V MMAs first.
+// With 128-key tiles P has buffers of its own and the two kinds interleave.
+template <bool kF8, int kBN>
 struct Cfg {
+  static_assert(kBN == 128 || (kBN == 192 && !kF8), "key tiles of 128 keys, or 192 with the bf16 cache");
   static constexpr int kHalves = kF8 ? 2 : 1;         // softmax warps per 32 rows
   static constexpr int kSoftmaxWarps = 4 * kHalves;
   static constexpr int kProducerWarp = kSoftmaxWarps, kMmaWarp = kSoftmaxWarps + 1, kGateWarp = kSoftmaxWarps + 2;
   static constexpr int kThreads = 32 * (kSoftmaxWarps + 3);
   static constexpr int kWarpArrivals = 2 * kSoftmaxWarps;  // p_full / q8_full: every softmax warp of both CTAs
+  static constexpr int kStages = kBN == 128 ? 4 : 3;     // ring stages (shared memory: 2 Q + stages <= 227 KB)
+  static constexpr uint32_t kKBox = (kBN / 2) * 128;     // one K box: kBN / 2 rows x 128 bytes
+  static constexpr uint32_t kKHalf = 2 * kKBox;          // this CTA's kBN / 2 keys x 128 d of a K tile
+  static constexpr uint32_t kVHalf = kBN * 64 * 2;       // kBN keys x this CTA's 64 d of a V tile
+  static constexpr uint32_t kStage = kKHalf + kVHalf;
+  static constexpr bool kPOverS = kBN != 128;
+  static constexpr uint32_t kColS = 0;                   // S buffer b at kColS + b * kBN
+  static constexpr uint32_t kColP = kPOverS ? 0u : 256u; // P buffer b at kColP + b * kPStride
+  static constexpr uint32_t kPStride = kPOverS ? kBN : 64u;
+  static constexpr uint32_t kColO = 384;
+  static_assert(2 * kBN <= 384 && kColO + kD <= tc::kTmemCols, "tensor-memory layout");
 };
+constexpr int kPairDoneBars = 4;          // pair_done[g % 4]: a waiter for group g holds up group g + 4
 constexpr uint32_t kGateBarrier = 1;  // named barrier of the MMA and gate warps (0 is __syncthreads)
 constexpr uint32_t kKHalf8 = 64 * 128;   // 8 KB: this CTA's 64 keys x 128 d of an E4M3 K tile
 constexpr uint32_t kVHalf8 = 64 * 128;   // 8 KB: this CTA's 64 d x 128 keys of an E4M3 V^T tile
 constexpr uint32_t kQ8Tile = 128 * 128;  // this CTA's 128 query rows as E4M3
 constexpr int kScaleSlots = 8;           // ring of per-tile scales of cached tiles (E4M3 kernel)
-static_assert(kStages == 4, "pair_done indexing assumes four stages");
 
-template <bool kF8>
+template <bool kF8, int kBN>
 struct SmemT {
+  using C = Cfg<kF8, kBN>;
+  static constexpr int kStages = C::kStages;
   static constexpr uint32_t kQ = 0;                // Q buffers 0 and 1 (this CTA's 128 rows)
   static constexpr uint32_t kRing = 2 * kQTile;    // stage s: [K half | V half]
-  static constexpr uint32_t kQ8 = kRing + kStages * kStage;  // E4M3 Q tile (kF8 only)
+  static constexpr uint32_t kQ8 = kRing + kStages * C::kStage;  // E4M3 Q tile (kF8 only)
   static constexpr uint32_t kScales = kQ8 + (kF8 ? kQ8Tile : 0u);  // ring of kScaleSlots x 16 B (kF8 only)
   static constexpr uint32_t kLX = kScales + (kF8 ? kScaleSlots * 16u : 0u);  // [2][128] fp32 partial row sums
   static constexpr uint32_t kBars = kLX + (kF8 ? 2u * 128u * 4u : 0u);
-  static constexpr int kQFull = 0, kQEmpty = 2, kStageFull = 4, kPairDone = 4 + kStages, kPFull = kPairDone + 4,
-                       kMmaDone = kPFull + 2, kQ8Full = kMmaDone + 1, kLXFull = kQ8Full + 1,
-                       kScaleFull = kLXFull + 1, kScaleEmpty = kScaleFull + kScaleSlots,
+  static constexpr int kQFull = 0, kQEmpty = 2, kStageFull = 4, kPairDone = 4 + kStages,
+                       kPFull = kPairDone + kPairDoneBars, kMmaDone = kPFull + 2, kQ8Full = kMmaDone + 1,
+                       kLXFull = kQ8Full + 1, kScaleFull = kLXFull + 1, kScaleEmpty = kScaleFull + kScaleSlots,
                        kNumBars = kScaleEmpty + kScaleSlots;
   static constexpr uint32_t kTmemHolder = kBars + 8 * kNumBars;
   static constexpr uint32_t kAbort = kTmemHolder + 4;
@@ -134,11 +151,38 @@ struct SmemT {
   static constexpr uint32_t kMaxDynamic = 232448;
   static constexpr uint32_t kDynamic = kUsed + 1024 < kMaxDynamic ? kUsed + 1024 : kMaxDynamic;
   static_assert(kUsed <= kMaxDynamic, "shared-memory layout too large");
+  static_assert(C::kStage % 1024 == 0 && C::kKBox % 1024 == 0, "swizzle atoms start on 1024-byte boundaries");
 };
-using Smem = SmemT<false>;
 
-// Phase parity of pair_done[g % 4] / stage_full[g % 4] for group g.
+// Key tiles of kBN keys: tile j of an item (range A first, then range B).
+template <int kBN>
+__device__ __forceinline__ tc::TileSrc tile_src(const Task& t, int na, int j) {
+  tc::TileSrc s;
+  if (j < na) {
+    s.row = t.a_row0 + j * kBN;
+    s.valid = min(kBN, t.a_len - j * kBN);
+    s.in_b = false;
+  } else {
+    const int jj = j - na;
+    s.row = t.b_row0 + jj * kBN;
+    s.valid = min(kBN, t.b_len - jj * kBN);
+    s.in_b = true;
+  }
+  return s;
+}
+template <int kBN>
+__device__ __forceinline__ int n_key_tiles(const Task& t, int& na) {
+  na = (t.a_len + kBN - 1) / kBN;
+  return na + (t.b_len + kBN - 1) / kBN;
+}
+
+// Phase parity of pair_done[g % 4] for group g.
 __device__ __forceinline__ uint32_t group_parity(int g) { return static_cast<uint32_t>(g >> 2) & 1u; }
+// Ring stage of group g and the phase parity of its stage_full barrier.
+template <int kStages>
+__device__ __forceinline__ int stage_of(int g) { return g % kStages; }
+template <int kStages>
+__device__ __forceinline__ uint32_t stage_parity(int g) { return static_cast<uint32_t>(g / kStages) & 1u; }
 
 // Bounded wait with cluster-scope acquire (barriers other CTAs arrive on).
 __device__ __forceinline__ bool wait_cl(uint32_t bar, uint32_t parity, const Ctl& c, int where) {
@@ -161,28 +205,31 @@ __device__ __forceinline__ bool wait_cl_warp(uint32_t bar, uint32_t parity, cons
 }
 }  // namespace tc2
 
-template <bool kF8>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThreads, 1)
+template <bool kF8, int kBN>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::kThreads, 1)
     attn_tc2_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_ka,
                     const __grid_constant__ CUtensorMap tm_va, const __grid_constant__ CUtensorMap tm_kb,
                     const __grid_constant__ CUtensorMap tm_vb, const AttnArgs args) {
   using namespace tc;
-  using tc2::kKBox;
-  using tc2::kKHalf;
   using tc2::kQTile;
-  using tc2::kStage;
-  using tc2::kStages;
-  using tc2::kVHalf;
-  using Cfg = tc2::Cfg<kF8>;
+  using Cfg = tc2::Cfg<kF8, kBN>;
+  constexpr uint32_t kKBox = Cfg::kKBox;
+  constexpr uint32_t kKHalf = Cfg::kKHalf;
+  constexpr uint32_t kVHalf = Cfg::kVHalf;
+  constexpr uint32_t kStage = Cfg::kStage;
+  constexpr int kStages = Cfg::kStages;
+  constexpr uint32_t kColS = Cfg::kColS, kColP = Cfg::kColP, kPStride = Cfg::kPStride, kColO = Cfg::kColO;
   constexpr int kWarpArrivals = Cfg::kWarpArrivals;
   using tc2::group_parity;
   using tc2::wait_cl;
   using tc2::wait_cl_warp;
   using tc2::kKHalf8;
   using tc2::kVHalf8;
-  using L = tc2::SmemT<kF8>;
+  using L = tc2::SmemT<kF8, kBN>;
   constexpr int D = tc2::kD;
-  constexpr uint32_t kIdescS = idesc_bf16_f32(256, 128, false);
+  auto stage_of = [](int g) -> int { return tc2::stage_of<kStages>(g); };
+  auto stage_parity = [](int g) -> uint32_t { return tc2::stage_parity<kStages>(g); };
+  constexpr uint32_t kIdescS = idesc_bf16_f32(256, kBN, false);
   constexpr uint32_t kIdescO = idesc_bf16_f32(256, D, true);
   constexpr uint32_t kIdesc8 = idesc_e4m3_f32(256, 128);  // S and O of cached tiles (N = 128 keys or d)
 
@@ -212,10 +259,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
       mbar_init(bar(L::kQEmpty + i), 1);
       mbar_init(bar(L::kPFull + i), kWarpArrivals);
     }
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(bar(L::kStageFull + s), 1);
-      mbar_init(bar(L::kPairDone + s), 1);
-    }
+    for (int s = 0; s < kStages; ++s) mbar_init(bar(L::kStageFull + s), 1);
+    for (int s = 0; s < tc2::kPairDoneBars; ++s) mbar_init(bar(L::kPairDone + s), 1);
     mbar_init(bar(L::kMmaDone), 1);
     mbar_init(bar(L::kQ8Full), kWarpArrivals);
     mbar_init(bar(L::kLXFull), Cfg::kSoftmaxWarps);
@@ -267,13 +312,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
       int head = 0, na = 0;
       // stage of group g: K tile kj (if kj >= 0) and V tile vj (if vj >= 0) of the item
       auto load_stage = [&](int kj, int vj) -> bool {
-        const int slot = g & (kStages - 1);
+        const int slot = stage_of(g);
         // the stage's previous group (g - kStages) must be complete
-        if (g >= kStages && !wait_one(bar(L::kPairDone + slot), group_parity(g - kStages), ctl, 2)) return false;
+        if (g >= kStages &&
+            !wait_one(bar(L::kPairDone + ((g - kStages) & 3)), group_parity(g - kStages), ctl, 2))
+          return false;
         const uint32_t dst = base + L::kRing + static_cast<uint32_t>(slot) * kStage;
         const uint32_t full = lbar(L::kStageFull + slot);
-        const TileSrc ks = tile_src(tk, na, kj >= 0 ? kj : 0);
-        const TileSrc vs = tile_src(tk, na, vj >= 0 ? vj : 0);
+        const TileSrc ks = tc2::tile_src<kBN>(tk, na, kj >= 0 ? kj : 0);
+        const TileSrc vs = tc2::tile_src<kBN>(tk, na, vj >= 0 ? vj : 0);
         const bool k8 = kF8 && kj >= 0 && ks.in_b, v8 = kF8 && vj >= 0 && vs.in_b;
         const uint32_t bytes =
             2 * ((kj >= 0 ? (k8 ? kKHalf8 : kKHalf) : 0u) + (vj >= 0 ? (v8 ? kVHalf8 : kVHalf) : 0u));
@@ -297,14 +344,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
           own_bytes[slot] = bytes / 2;
           if (k8) {  // E4M3 keys [64 r, 64 r + 64): one box of 64 rows x 128 bytes
             tma_load_2d_pair(dst, &tm_kb, full, head * D, ks.row + 64 * static_cast<int>(rank));
-          } else if (kj >= 0) {  // keys [64 r, 64 r + 64) of the tile, both head-dim boxes
+          } else if (kj >= 0) {  // keys [kBN/2 r, kBN/2 (r + 1)) of the tile, both head-dim boxes
             const void* map = ks.in_b ? &tm_kb : &tm_ka;
             for (int ch = 0; ch < 2; ++ch)
-              tma_load_2d_pair(dst + ch * kKBox, map, full, head * D + ch * 64, ks.row + 64 * static_cast<int>(rank));
+              tma_load_2d_pair(dst + ch * kKBox, map, full, head * D + ch * 64,
+                               ks.row + (kBN / 2) * static_cast<int>(rank));
           }
           if (v8) {  // E4M3 V^T rows d in [64 r, 64 r + 64), all 128 keys
             tma_load_2d_pair(dst + kKHalf, &tm_vb, full, vs.row, head * D + 64 * static_cast<int>(rank));
-          } else if (vj >= 0) {  // head-dim columns [64 r, 64 r + 64) of all 128 keys
+          } else if (vj >= 0) {  // head-dim columns [64 r, 64 r + 64) of all kBN keys
             const void* map = vs.in_b ? &tm_vb : &tm_va;
             tma_load_2d_pair(dst + kKHalf, map, full, head * D + 64 * static_cast<int>(rank), vs.row);
           }
@@ -314,7 +362,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
       };
       for (int item = cluster; item < args.n_items; item += n_clusters) {
         decode_item(args, item, tk, head);
-        const int nkv = n_key_tiles(tk, na);
+        const int nkv = tc2::n_key_tiles<kBN>(tk, na);
         if (nkv == 0) continue;
         {  // this CTA's 128 query rows into Q buffer qi % 2
           const int b = qi & 1;
@@ -354,13 +402,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
     if (leader) {
       // descriptors of stage 0 (stage s: + s * kStage / 16) and of Q buffer 0
       const uint64_t kd0 = sdesc_sw128(base + L::kRing, 16, 1024);
-      const uint64_t vd0 = sdesc_sw128(base + L::kRing + kKHalf, kBoxBytes, 1024);
+      const uint64_t vd0 = sdesc_sw128(base + L::kRing + kKHalf, Cfg::kVHalf, 1024);
       const uint64_t qdesc0 = sdesc_sw128(base + L::kQ, 16, 1024);
       // E4M3 operands: Q8 (128 rows x 128 B), K8 half (64 rows x 128 B), V^T half (64 d x 128 B); a
       // K = 32 step advances 32 bytes inside the swizzle atom
       const uint64_t q8d = sdesc_sw128(base + L::kQ8, 16, 1024);
       const uint64_t vd80 = sdesc_sw128(base + L::kRing + kKHalf, 16, 1024);
-      // S step kk: A = Q (128-row boxes of 16 KB), B = this CTA's 64 keys (64-row boxes of 8 KB)
+      // S step kk: A = Q (128-row boxes of 16 KB), B = this CTA's kBN / 2 keys (boxes of kBN / 2 rows)
       auto q_off = [](int kk) -> uint64_t {
         return (static_cast<uint32_t>(kk >> 2) * kBoxBytes + static_cast<uint32_t>(kk & 3) * 32u) >> 4;
       };
@@ -373,19 +421,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
         Task tk;
         int head, na;
         decode_item(args, item, tk, head);
-        const int nkv = n_key_tiles(tk, na);
+        const int nkv = tc2::n_key_tiles<kBN>(tk, na);
         if (nkv == 0) continue;
         const int qb = qi & 1;
         const uint64_t qd = qdesc0 + ((static_cast<uint32_t>(qb) * kQTile) >> 4);
         // groups G, G + 1: S_0, S_1 (the gate warp has seen the Q tile and stage g land)
         for (int n = 0; n < 2; ++n, ++g) {
           if (bar_red_or(tc2::kGateBarrier, 64, false)) goto mma_done;
-          const int slot = g & (kStages - 1);
+          const int slot = stage_of(g);
           if (lane == 0) {
             if (n < nkv) {
               tc_fence_after();
               const uint64_t kd = kd0 + static_cast<uint64_t>(slot) * (kStage >> 4);
-              const uint32_t d_s = tmem + kColS + (static_cast<uint32_t>((t0 + n) & 1) << 7);
+              const uint32_t d_s = tmem + kColS + static_cast<uint32_t>((t0 + n) & 1) * kBN;
               if (kF8 && n >= na) {
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk)
@@ -397,7 +445,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
               }
               if (n == nkv - 1) tc2_commit_mc(bar(L::kQEmpty + qb), 3);
             }
-            tc2_commit_mc(bar(L::kPairDone + slot), 3);
+            tc2_commit_mc(bar(L::kPairDone + (g & 3)), 3);
           }
           issued = true;
           __syncwarp();
@@ -409,18 +457,26 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
           if (lane == 0) {
             const int t = t0 + j;
             tc_fence_after();
-            const int slot = g & (kStages - 1);
+            const int slot = stage_of(g);
             const uint64_t soff = static_cast<uint64_t>(slot) * (kStage >> 4);
             const uint64_t vd = vd0 + soff;
-            const uint32_t a_p = tmem + kColP + (static_cast<uint32_t>(t & 1) << 6);
+            const uint32_t a_p = tmem + kColP + static_cast<uint32_t>(t & 1) * kPStride;
             const uint32_t acc0 = j > 0 ? 1u : 0u;
             const bool pv8 = kF8 && j >= na;      // P_j V_j on E4M3 operands
             const bool s8 = kF8 && j + 2 >= na;   // S_j+2 on E4M3 operands
             const uint64_t vd8 = vd80 + soff;
             if (j + 2 < nkv) {
               const uint64_t kd = kd0 + soff;
-              const uint32_t d_s = tmem + kColS + (static_cast<uint32_t>(t & 1) << 7);
-              if (!s8) {
+              const uint32_t d_s = tmem + kColS + static_cast<uint32_t>(t & 1) * kBN;
+              if (!s8 && Cfg::kPOverS) {
+                // S_j+2 overwrites P_j: every P.V MMA of the group goes first
+#pragma unroll
+                for (int kk = 0; kk < kBN / 16; ++kk)
+                  tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, kk > 0 ? 1u : acc0);
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk)
+                  tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
+              } else if (!s8) {
 #pragma unroll
                 for (int kk = 0; kk < 8; ++kk) {
                   tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, kk > 0 ? 1u : acc0);
@@ -447,10 +503,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
                 tc2_mma_ts_f8(tmem + kColO, a_p + 8u * kk, vd8 + ((32u * kk) >> 4), kIdesc8, kk > 0 ? 1u : acc0);
             } else {
 #pragma unroll
-              for (int kk = 0; kk < 8; ++kk)
+              for (int kk = 0; kk < kBN / 16; ++kk)
                 tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, kk > 0 ? 1u : acc0);
             }
-            tc2_commit_mc(bar(L::kPairDone + slot), 3);
+            tc2_commit_mc(bar(L::kPairDone + (g & 3)), 3);
           }
           __syncwarp();
         }
@@ -474,14 +530,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
         Task tk;
         int head, na;
         decode_item(args, item, tk, head);
-        const int nkv = n_key_tiles(tk, na);
+        const int nkv = tc2::n_key_tiles<kBN>(tk, na);
         if (nkv == 0) continue;
         // the first cached tile's S also needs the E4M3 Q tile of both CTAs
         const bool q8 = kF8 && nkv > na;
         const uint32_t q8_parity = static_cast<uint32_t>(q8i) & 1u;
         bool ok = wait_cl_warp(bar(L::kQFull + (qi & 1)), static_cast<uint32_t>(qi >> 1) & 1u, ctl, 3);
         for (int n = 0; n < 2; ++n, ++g) {
-          ok = ok && wait_cl_warp(bar(L::kStageFull + (g & (kStages - 1))), group_parity(g), ctl, 4);
+          ok = ok && wait_cl_warp(bar(L::kStageFull + stage_of(g)), stage_parity(g), ctl, 4);
           if (q8 && n == na) ok = ok && wait_cl_warp(bar(L::kQ8Full), q8_parity, ctl, 14);
           if (bar_red_or(tc2::kGateBarrier, 64, !ok)) goto gate_done;
         }
@@ -507,9 +563,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
     // and take the same rescale decisions; their partial row sums meet in the
     // epilogue through shared memory.
     constexpr int kH = Cfg::kHalves;
-    constexpr int kC = 128 / kH;  // key columns and O columns of this thread
+    constexpr int kC = kBN / kH;  // key columns of this thread
+    constexpr int kOC = D / kH;   // O columns of this thread
     const int quarter = warp & 3, hh = warp >> 2;
-    const int col0 = hh * kC;
+    const int col0 = hh * kC, ocol0 = hh * kOC;
     const int trow = quarter * 32 + lane;                  // row within this CTA's 128 rows (= TMEM lane)
     const int prow = 128 * static_cast<int>(rank) + trow;  // row within the item
     const uint32_t lane_off = static_cast<uint32_t>(quarter * 32) << 16;
@@ -529,14 +586,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
       int head;
       decode_item(args, item, tk, head);
       int na;
-      const int nkv = n_key_tiles(tk, na);
+      const int nkv = tc2::n_key_tiles<kBN>(tk, na);
       const bool row_ok = prow < tk.q_rows;
       const int64_t grow = static_cast<int64_t>(tk.q_row0) + prow;
-      __nv_bfloat16* orow = args.out + grow * args.row_stride + static_cast<int64_t>(head) * D + col0;
+      __nv_bfloat16* orow = args.out + grow * args.row_stride + static_cast<int64_t>(head) * D + ocol0;
       if (nkv == 0) {
         if (row_ok) {
           uint4 z = make_uint4(0, 0, 0, 0);
-          for (int c = 0; c < kC / 8; ++c) reinterpret_cast<uint4*>(orow)[c] = z;
+          for (int c = 0; c < kOC / 8; ++c) reinterpret_cast<uint4*>(orow)[c] = z;
           if (args.lse && hh == 0) args.lse[grow * args.num_heads + head] = -INFINITY;
         }
         continue;
@@ -593,7 +650,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
       }
       for (int j = 0; j < nkv; ++j, ++t) {
         const int b = t & 1;
-        const TileSrc src = tile_src(tk, na, j);
+        const TileSrc src = tc2::tile_src<kBN>(tk, na, j);
         // per-tile constants: u = c * s + shift is the shifted scaled score, the
         // weight written is exp2(u - m + wshift), the tile adds lscale * sum to l
         const bool t8 = kF8 && j >= na;
@@ -618,31 +675,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
         // S_j is ready and P buffer b is free once group G + j is complete
         if (!wait_group(G + j, 8)) goto softmax_done;
         tc_fence_after();
-        const uint32_t t_s = tmem + lane_off + kColS + 128u * b;
+        const uint32_t t_s = tmem + lane_off + kColS + static_cast<uint32_t>(kBN) * b;
         // this thread's columns of S in s[]; with two halves, the other half's
         // maximum in m_other
         float s[kC];
         float m_other = -INFINITY;
         if constexpr (kH == 1) {
-          uint32_t r0[32], r1[32], r2[32], r3[32];
-          tmem_ld32(t_s + 0u, r0);
-          tmem_ld32(t_s + 32u, r1);
-          tmem_ld32(t_s + 64u, r2);
-          tmem_ld32(t_s + 96u, r3);
-          tmem_wait_ld(r0);
-          tmem_wait_ld(r1);
-          tmem_wait_ld(r2);
-          tmem_wait_ld(r3);
+          uint32_t r[kC / 32][32];
 #pragma unroll
-          for (int c = 0; c < 32; ++c) {
-            s[c] = __uint_as_float(r0[c]);
-            s[32 + c] = __uint_as_float(r1[c]);
-            s[64 + c] = __uint_as_float(r2[c]);
-            s[96 + c] = __uint_as_float(r3[c]);
-          }
-          if (src.valid < 128) {  // keys past the end of the range
+          for (int k = 0; k < kC / 32; ++k) tmem_ld32(t_s + 32u * k, r[k]);
 #pragma unroll
-            for (int c = 0; c < 128; ++c)
+          for (int k = 0; k < kC / 32; ++k) tmem_wait_ld(r[k]);
+#pragma unroll
+          for (int k = 0; k < kC / 32; ++k)
+#pragma unroll
+            for (int c = 0; c < 32; ++c) s[32 * k + c] = __uint_as_float(r[k][c]);
+          if (src.valid < kBN) {  // keys past the end of the range
+#pragma unroll
+            for (int c = 0; c < kC; ++c)
               if (c >= src.valid) s[c] = -INFINITY;
           }
         } else {
@@ -694,7 +744,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
             for (int c = 3; c < 31; c += 2) mx[k] = fmax3(mx[k], s[32 * k + c], s[32 * k + c + 1]);
             mx[k] = fmaxf(mx[k], s[32 * k + 31]);
           }
-          if constexpr (kChains == 4)
+          if constexpr (kChains == 6)
+            return fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]), -INFINITY);
+          else if constexpr (kChains == 4)
             return fmax3(mx[0], mx[1], fmaxf(mx[2], mx[3]));
           else
             return fmax3(mx[0], mx[1], m_other);
@@ -708,9 +760,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
           const f32x2 alpha2 = make_f32x2(alpha, alpha);
           m_run = m_new;
           l_run *= alpha;
-          const uint32_t t_o = tmem + lane_off + kColO + static_cast<uint32_t>(col0);
+          const uint32_t t_o = tmem + lane_off + kColO + static_cast<uint32_t>(ocol0);
 #pragma unroll
-          for (int cc = 0; cc < kC / 16; ++cc) {
+          for (int cc = 0; cc < kOC / 16; ++cc) {
             uint32_t o[16];
             tmem_ld16(t_o + 16u * cc, o);
             tmem_wait_ld(o);
@@ -729,7 +781,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
         // P = exp2(c * S + shift - m) into P buffer b: bf16 pairs (32 keys = 16
         // columns at a time), or for a cached tile E4M3 quads (32 keys = 8
         // columns); returns this thread's sum of the weights written
-        const uint32_t t_p = tmem + lane_off + kColP + 64u * b;
+        const uint32_t t_p = tmem + lane_off + kColP + kPStride * b;
         auto write_p = [&]() -> float {
           const float bias = (kF8 ? shift + wshift : 0.f) - m_run;
           const f32x2 negm = make_f32x2(bias, bias);
@@ -789,7 +841,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
         // the MMA thread waits only for P: the leader's warp 0 first makes
         // sure that the stage of P_j V_j's group (G + j + 2) has landed
         if (leader && warp == 0 &&
-            !wait_warp(bar(L::kStageFull + ((G + j + 2) & (kStages - 1))), group_parity(G + j + 2), ctl, 13))
+            !wait_warp(bar(L::kStageFull + stage_of(G + j + 2)), stage_parity(G + j + 2), ctl, 13))
           goto softmax_done;
         tmem_wait_st();
         tc_fence_before();
@@ -810,13 +862,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
           l_tot = l_run + lx[(1 - hh) * 128 + trow];
         }
         const float inv_l = kF8 ? s_ref / l_tot : 1.0f / l_tot;
-        const uint32_t t_o = tmem + lane_off + kColO + static_cast<uint32_t>(col0);
+        const uint32_t t_o = tmem + lane_off + kColO + static_cast<uint32_t>(ocol0);
         if (tk.part > 0) {
           // a part of a split item: O / l in fp32 and m + log l to its workspace slot
           const int64_t prow_ws = static_cast<int64_t>(tk.part - 1) * args.rows_per_task + prow;
-          float4* dst = reinterpret_cast<float4*>(args.part_o + prow_ws * D + col0);
+          float4* dst = reinterpret_cast<float4*>(args.part_o + prow_ws * D + ocol0);
 #pragma unroll
-          for (int cc = 0; cc < kC / 32; ++cc) {
+          for (int cc = 0; cc < kOC / 32; ++cc) {
             uint32_t o[32];
             tmem_ld32(t_o + 32u * cc, o);
             tmem_wait_ld(o);
@@ -833,9 +885,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
           G += nkv + 2;
           continue;
         }
-        uint32_t packed[kC / 2];
+        uint32_t packed[kOC / 2];
 #pragma unroll
-        for (int cc = 0; cc < kC / 32; ++cc) {
+        for (int cc = 0; cc < kOC / 32; ++cc) {
           uint32_t o[32];
           tmem_ld32(t_o + 32u * cc, o);
           tmem_wait_ld(o);
@@ -850,7 +902,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8>::kThre
         if (row_ok) {
           uint4* dst = reinterpret_cast<uint4*>(orow);
 #pragma unroll
-          for (int c = 0; c < kC / 8; ++c)
+          for (int c = 0; c < kOC / 8; ++c)
             dst[c] = make_uint4(packed[4 * c], packed[4 * c + 1], packed[4 * c + 2], packed[4 * c + 3]);
           if (args.lse && hh == 0)
             args.lse[grow * args.num_heads + head] = (m_run + log2f(l_tot)) * 0.69314718055994530942f;

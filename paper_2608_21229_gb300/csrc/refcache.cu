@@ -58,8 +58,8 @@ struct DeviceInfo {
   bool checked = false;
   bool ok = false;
   int num_sms = 0;
-  bool attr_set[6] = {false, false, false, false, false, false};
-  int max_clusters[2] = {0, 0};  // CTA pairs of attn_tc2_kernel<false>, <true> that fit at once
+  bool attr_set[7] = {false, false, false, false, false, false, false};
+  int max_clusters[3] = {0, 0, 0};  // CTA pairs of each attn_tc2_kernel variant that fit at once
 };
 DeviceInfo g_dev[kMaxDevices];
 std::mutex g_dev_mu;
@@ -213,44 +213,50 @@ int launch_tc(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info,
   return REFCACHE_OK;
 }
 
-// CTA pairs of the head-dim-128 kernel (bf16 key range B, or E4M3 with kF8)
-// that run at once on this device (the persistent grid); sets the kernel's
-// shared-memory attribute on first use.
-template <bool kF8>
+// Keys per tile of the head-dim-128 pair kernel: 192 for the bf16 cache
+// (REFCACHE_KERNEL_TCGEN05), 128 for the E4M3 cache and for
+// REFCACHE_KERNEL_TCGEN05_K128.
+int tc2_tile(bool f8) { return f8 || g_kernel.load() == REFCACHE_KERNEL_TCGEN05_K128 ? 128 : 192; }
+
+// CTA pairs of the head-dim-128 kernel (bf16 key range B, or E4M3 with kF8;
+// kBN keys per tile) that run at once on this device (the persistent grid);
+// sets the kernel's shared-memory attribute on first use.
+template <bool kF8, int kBN>
 int tc2_clusters(DeviceInfo* info, int* clusters_out) {
-  constexpr uint32_t smem = rc::tc2::SmemT<kF8>::kDynamic;
-  const int key = kF8 ? 5 : 4;
+  constexpr uint32_t smem = rc::tc2::SmemT<kF8, kBN>::kDynamic;
+  const int variant = kF8 ? 1 : kBN == 128 ? 0 : 2;
+  const int key = 4 + variant;
   if (!info->attr_set[key]) {
     cudaError_t e =
-        cudaFuncSetAttribute(rc::attn_tc2_kernel<kF8>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        cudaFuncSetAttribute(rc::attn_tc2_kernel<kF8, kBN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_tc2_kernel)");
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3(2 * static_cast<unsigned>(info->num_sms / 2), 1, 1);
-    cfg.blockDim = dim3(rc::tc2::Cfg<kF8>::kThreads, 1, 1);
+    cfg.blockDim = dim3(rc::tc2::Cfg<kF8, kBN>::kThreads, 1, 1);
     cfg.dynamicSmemBytes = smem;
     int clusters = 0;
-    e = cudaOccupancyMaxActiveClusters(&clusters, rc::attn_tc2_kernel<kF8>, &cfg);
+    e = cudaOccupancyMaxActiveClusters(&clusters, rc::attn_tc2_kernel<kF8, kBN>, &cfg);
     if (e != cudaSuccess || clusters < 1) clusters = info->num_sms / 2;
-    info->max_clusters[kF8 ? 1 : 0] = clusters;
+    info->max_clusters[variant] = clusters;
     info->attr_set[key] = true;
   }
-  *clusters_out = info->max_clusters[kF8 ? 1 : 0];
+  *clusters_out = info->max_clusters[variant];
   return REFCACHE_OK;
 }
 
 // The CTA-pair kernel (head_dim 128): grid = 2 x the clusters that fit at once.
-template <bool kF8>
+template <bool kF8, int kBN>
 int launch_tc2(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info, cudaStream_t s) {
-  constexpr uint32_t smem = rc::tc2::SmemT<kF8>::kDynamic;
+  constexpr uint32_t smem = rc::tc2::SmemT<kF8, kBN>::kDynamic;
   int max_clusters = 0;
-  int rc = tc2_clusters<kF8>(info, &max_clusters);
+  int rc = tc2_clusters<kF8, kBN>(info, &max_clusters);
   if (rc) return rc;
   const int clusters = std::min(a.n_items, max_clusters);
   // a programmatic dependent of the stream's previous kernel: its prologue
   // (barriers, tensor memory) overlaps that kernel's tail
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(2 * static_cast<unsigned>(clusters), 1, 1);
-  cfg.blockDim = dim3(rc::tc2::Cfg<kF8>::kThreads, 1, 1);
+  cfg.blockDim = dim3(rc::tc2::Cfg<kF8, kBN>::kThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
@@ -258,7 +264,8 @@ int launch_tc2(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, rc::attn_tc2_kernel<kF8>, maps[0], maps[1], maps[2], maps[3], maps[4], a);
+  cudaError_t e =
+      cudaLaunchKernelEx(&cfg, rc::attn_tc2_kernel<kF8, kBN>, maps[0], maps[1], maps[2], maps[3], maps[4], a);
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "attn_tc2_kernel launch");
   return REFCACHE_OK;
@@ -373,20 +380,23 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
     if (rc) return rc;
     return D == 64 ? launch_mma<64>(a, info, s) : launch_mma<128>(a, info, s);
   }
-  // K tiles of the CTA-pair kernel are loaded as two 64-row halves
-  const uint32_t k_rows = D == 128 ? 64 : 128;
+  // Key tiles of the CTA-pair kernel: each CTA loads half of a K tile (two
+  // boxes of tile / 2 rows) and a V box of the whole tile; head dim 64 loads
+  // 128-row boxes.
+  const uint32_t tile = D == 128 ? static_cast<uint32_t>(tc2_tile(f8 != nullptr)) : 128u;
+  const uint32_t k_rows = D == 128 ? tile / 2 : 128u, v_rows = tile;
   CUtensorMap maps[5];
   int rc;
   if ((rc = make_tmap(&maps[0], op.q, op.q_rows, H, D)) != 0) return rc;
   if ((rc = make_tmap(&maps[1], op.ka, op.a_rows, H, D, k_rows)) != 0) return rc;
-  if ((rc = make_tmap(&maps[2], op.va, op.a_rows, H, D)) != 0) return rc;
+  if ((rc = make_tmap(&maps[2], op.va, op.a_rows, H, D, v_rows)) != 0) return rc;
   if (f8) {
     if ((rc = make_tmap_u8(&maps[3], f8->k8, static_cast<int64_t>(H) * D, f8->rows_pad)) != 0) return rc;
     if ((rc = make_tmap_u8(&maps[4], f8->vt8, f8->rows_pad, static_cast<int64_t>(H) * D)) != 0) return rc;
     a.b_scales = f8->scales;
   } else if (op.kb && op.b_rows > 0) {
     if ((rc = make_tmap(&maps[3], op.kb, op.b_rows, H, D, k_rows)) != 0) return rc;
-    if ((rc = make_tmap(&maps[4], op.vb, op.b_rows, H, D)) != 0) return rc;
+    if ((rc = make_tmap(&maps[4], op.vb, op.b_rows, H, D, v_rows)) != 0) return rc;
   } else {
     maps[3] = maps[1];
     maps[4] = maps[2];
@@ -403,7 +413,9 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
     a.part_o = il->part_o;
     a.part_lse = il->part_lse;
   }
-  if ((rc = f8 ? launch_tc2<true>(maps, a, info, s) : launch_tc2<false>(maps, a, info, s)) != 0) return rc;
+  rc = f8 ? launch_tc2<true, 128>(maps, a, info, s)
+          : tile == 128 ? launch_tc2<false, 128>(maps, a, info, s) : launch_tc2<false, 192>(maps, a, info, s);
+  if (rc) return rc;
   if (copy && (rc = launch_copy(*copy, info, s, true)) != 0) return rc;
   if (il && il->n_jobs > 0) {
     cudaLaunchConfig_t cfg{};
@@ -429,7 +441,7 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
 // of the persistent grid, the items of that round are split by key tiles into
 // s parts each (s chosen so that the parts fill the clusters best), which run
 // after the whole items; their results are merged by combine jobs.
-void plan_items(const std::vector<Task>& tasks, int H, int clusters, std::vector<Task>* items,
+void plan_items(const std::vector<Task>& tasks, int H, int clusters, int tile, std::vector<Task>* items,
                 std::vector<CombineJob>* jobs, int* n_parts) {
   items->clear();
   jobs->clear();
@@ -455,7 +467,7 @@ void plan_items(const std::vector<Task>& tasks, int H, int clusters, std::vector
     Task t = tasks[static_cast<size_t>(i % static_cast<int64_t>(tasks.size()))];
     t.head = h;
     t.part = 0;
-    const int na = (t.a_len + 127) / 128, nb = (t.b_len + 127) / 128, nkv = na + nb;
+    const int na = (t.a_len + tile - 1) / tile, nb = (t.b_len + tile - 1) / tile, nkv = na + nb;
     const int s_here = std::min(best_s, nkv / 4);  // parts of at least four key tiles
     if (i < n_whole || s_here < 2) {
       items->push_back(t);
@@ -473,11 +485,11 @@ void plan_items(const std::vector<Task>& tasks, int H, int clusters, std::vector
       Task p = t;
       // tiles [j0, j1) of the item's key list (range A, then range B)
       const int a0 = std::min(j0, na), a1 = std::min(j1, na);
-      p.a_row0 = t.a_row0 + 128 * a0;
-      p.a_len = a1 > a0 ? std::min(t.a_len - 128 * a0, 128 * (a1 - a0)) : 0;
+      p.a_row0 = t.a_row0 + tile * a0;
+      p.a_len = a1 > a0 ? std::min(t.a_len - tile * a0, tile * (a1 - a0)) : 0;
       const int b0 = std::max(j0, na) - na, b1 = std::max(j1, na) - na;
-      p.b_row0 = t.b_row0 + 128 * b0;
-      p.b_len = b1 > b0 ? std::min(t.b_len - 128 * b0, 128 * (b1 - b0)) : 0;
+      p.b_row0 = t.b_row0 + tile * b0;
+      p.b_len = b1 > b0 ? std::min(t.b_len - tile * b0, tile * (b1 - b0)) : 0;
       p.part = ++*n_parts;
       parts.push_back(p);
     }
@@ -675,14 +687,18 @@ int check_ptrs(std::initializer_list<const void*> ps, int64_t rows, const char* 
 // only -- not on the other requests of the batch, nor on the device's SM count
 // -- and the cached block is reproduced bit for bit (Sec. 3.3).
 int plan_split_items(refcache* h, DeviceInfo* info, const std::vector<Task>& st) {
+  // planned for the step kernel selected now (key tiles of tc2_tile(); the
+  // parts stay correct, only less even, if another tile size runs them)
+  const bool f8 = h->f8 && h->rows_pad > 0;
+  const int tile = tc2_tile(f8);
   int clusters = 0;
-  int rc = tc2_clusters<false>(info, &clusters);
+  int rc = f8 ? tc2_clusters<true, 128>(info, &clusters)
+              : tile == 128 ? tc2_clusters<false, 128>(info, &clusters) : tc2_clusters<false, 192>(info, &clusters);
   if (rc) return rc;
-  if (h->f8 && h->rows_pad > 0 && (rc = tc2_clusters<true>(info, &clusters)) != 0) return rc;
   std::vector<Task> si;
   std::vector<CombineJob> sj;
   int parts = 0;
-  plan_items(st, h->H, clusters, &si, &sj, &parts);
+  plan_items(st, h->H, clusters, tile, &si, &sj, &parts);
   const int rows = task_rows(h->D);
   size_t off = 0;
   const size_t o_si = off;
@@ -846,7 +862,7 @@ int refcache_call_launches(refcache_t* h, int call) {
   const int n_tasks = call == 0 ? h->n_build : h->n_step;
   const int cache_write = call == 0 && (h->n_copy > 0 || h->n_qtiles > 0) ? 1 : 0;
   if (n_tasks == 0) return cache_write;
-  const bool tc = g_kernel.load() == REFCACHE_KERNEL_TCGEN05;
+  const bool tc = g_kernel.load() != REFCACHE_KERNEL_MMA_SYNC;
   const bool combine = call == 1 && tc && h->step_items.items && h->step_items.n_jobs > 0;
   return cache_write + 1 + (combine ? 1 : 0);
 }
@@ -1041,7 +1057,8 @@ int refcache_status(void* stream) {
 uint64_t refcache_set_wait_timeout_ns(uint64_t ns) { return g_timeout_ns.exchange(ns ? ns : 1); }
 
 int refcache_set_kernel(int kernel) {
-  if (kernel != REFCACHE_KERNEL_TCGEN05 && kernel != REFCACHE_KERNEL_MMA_SYNC)
+  if (kernel != REFCACHE_KERNEL_TCGEN05 && kernel != REFCACHE_KERNEL_MMA_SYNC &&
+      kernel != REFCACHE_KERNEL_TCGEN05_K128)
     return fail(REFCACHE_ERR_INVALID_ARG, "unknown kernel %d", kernel);
   return g_kernel.exchange(kernel);
 }

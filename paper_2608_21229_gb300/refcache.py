@@ -23,7 +23,7 @@ ERR_OOM = -5
 ERR_TIMEOUT = -6
 
 MASK_MODES = {"beyond": 0, "beyond_alt": 1, "isolated": 2}
-KERNELS = {"tcgen05": 0, "mma_sync": 1}
+KERNELS = {"tcgen05": 0, "mma_sync": 1, "tcgen05_k128": 2}
 CACHE_DTYPES = {"bf16": 0, "fp8": 0x100}  # REFCACHE_CACHE_FP8: E4M3 codes with per-tile scales
 
 EXPORTED = (

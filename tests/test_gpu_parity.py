@@ -17,7 +17,7 @@ import parity_utils as pu
 
 pytestmark = pytest.mark.gpu
 
-KERNELS = ["tcgen05", "mma_sync"]
+KERNELS = ["tcgen05", "tcgen05_k128", "mma_sync"]
 
 
 @pytest.fixture(scope="module", autouse=True)
