@@ -54,8 +54,8 @@
  *     with programmatic stream serialization after a library call must
  *     therefore wait for its grid dependencies (griddepcontrol.wait) before it
  *     reads the library's outputs; ordinary launches need nothing.
- *   - refcache_build and step_attention only launch kernels (no allocation,
- *     no copy), so they can be captured in a CUDA graph and replayed, once a
+ *   - refcache_build, refcache_build_in_slot and step_attention only launch
+ *     kernels (no allocation, no copy), so they can be captured in a CUDA graph and replayed, once a
  *     first call on the device has run outside the capture (the kernels'
  *     attributes are set on first use).  full_attention is not capturable
  *     (it copies its work list from host memory).
@@ -199,11 +199,12 @@ REFCACHE_API int refcache_fp8_ptr(refcache_t* cache, int layer, void** k8, void*
 REFCACHE_API int refcache_layer_built(refcache_t* cache, int layer);
 
 /*
- * Number of kernels one refcache_build (call = 0) or step_attention (call = 1)
- * on this cache launches with the kernel family currently selected
- * (refcache_set_kernel): the attention kernel, the cache write (build, when
- * there are cached rows: a copy, or the E4M3 quantisation) and the combine of
- * split items (when the cache's work list has any).  < 0 on error.
+ * Number of kernels one refcache_build (call = 0), step_attention (call = 1)
+ * or refcache_build_in_slot (call = 2) on this cache launches with the kernel
+ * family currently selected (refcache_set_kernel): the attention kernel, the
+ * cache write (refcache_build, when there are cached rows: a copy, or the
+ * E4M3 quantisation) and the combine of split items (step_attention, when the
+ * cache's work list has any).  < 0 on error.
  */
 REFCACHE_API int refcache_call_launches(refcache_t* cache, int call);
 
@@ -219,6 +220,31 @@ REFCACHE_API int refcache_call_launches(refcache_t* cache, int call);
 REFCACHE_API int refcache_build(refcache_t* cache, int layer, const void* q_static, const void* k_static,
                    const void* v_static, void* o_static, float* lse_static, float softmax_scale,
                    void* stream);
+
+/*
+ * The static prefill of one layer for a caller that projects the cached rows'
+ * K and V straight into the cache (the zero-copy path of Sec. 3.3: only R's
+ * K/V are kept, so they may be written where they are kept): before the call
+ * the layer's slots (refcache_kv_ptr) must hold the cached rows' K and V --
+ * R, or [ST; R] in REFCACHE_MASK_BEYOND_ALT -- of every request, in the
+ * slot's row order.  Computes what refcache_build computes (rows [ST; R] over
+ * keys [ST; R] under the cache's mask mode) and marks the layer built, but
+ * reads R's keys and values from the slots and launches no cache write.
+ *   q_static: [cu_static[batch], H, d] bf16, each request's [ST; R] queries.
+ *   k_anchor, v_anchor: [sum n_anchor, H, d] bf16, the anchors' K and V,
+ *     request b's n_anchor[b] rows after request b-1's; NULL when there are
+ *     no anchor rows, and ignored (may be NULL) in REFCACHE_MASK_BEYOND_ALT,
+ *     whose slots hold the anchors too.
+ *   o_static / lse_static as in refcache_build.
+ * The keys are tiled from the anchors and from R separately, so the outputs
+ * equal refcache_build's up to the rounding order of the sums, and repeated
+ * calls on the same inputs give the same bytes.  The slots are only read.
+ * REFCACHE_ERR_UNSUPPORTED for an E4M3 cache (REFCACHE_CACHE_FP8), which
+ * refcache_build writes from bf16 K and V.
+ */
+REFCACHE_API int refcache_build_in_slot(refcache_t* cache, int layer, const void* q_static, const void* k_anchor,
+                                        const void* v_anchor, void* o_static, float* lse_static, float softmax_scale,
+                                        void* stream);
 
 /*
  * One denoising step of one layer (App. C: [LT, X_t] queries over

@@ -525,6 +525,11 @@ struct refcache {
   bool owns = false;
   Task* d_build = nullptr;
   int n_build = 0;
+  // refcache_build_in_slot: the prefill over the cached rows already in the
+  // slot (key range B) and the anchors given apart (key range A)
+  Task* d_build_slot = nullptr;
+  int n_build_slot = 0;
+  int64_t anchor_rows = 0;
   Task* d_step = nullptr;
   int n_step = 0;
   CopySeg* d_copy = nullptr;
@@ -556,7 +561,7 @@ size_t fp8_layer_bytes(int64_t rows_pad, int H, int D) {
 
 int cache_plan(int num_layers, int mode_flags, const refcache_segments_t* seg, refcache* h,
                std::vector<Task>* build_tasks, std::vector<Task>* step_tasks, std::vector<CopySeg>* copies,
-               std::vector<QuantTile>* qtiles, size_t* total_bytes) {
+               std::vector<QuantTile>* qtiles, std::vector<Task>* slot_tasks, size_t* total_bytes) {
   if (!seg) return fail(REFCACHE_ERR_INVALID_ARG, "seg is NULL");
   if (num_layers < 1) return fail(REFCACHE_ERR_INVALID_ARG, "num_layers must be >= 1");
   const bool f8 = (mode_flags & REFCACHE_CACHE_FP8) != 0;
@@ -603,8 +608,9 @@ int cache_plan(int num_layers, int mode_flags, const refcache_segments_t* seg, r
   }
   if (off8[B] > max_rows) return fail(REFCACHE_ERR_INVALID_ARG, "cache rows too large");
   const int tr = task_rows(D);
-  std::vector<Task> bt, st;
+  std::vector<Task> bt, st, bs;
   std::vector<CopySeg> cp;
+  int a0 = 0;  // first row of request b's anchors in the anchor tensors of refcache_build_in_slot
   for (int b = 0; b < B; ++b) {
     const int s0 = seg->cu_static[b], ns = seg->cu_static[b + 1] - s0, na = seg->n_anchor[b];
     const int l0 = seg->cu_live[b], nl = seg->cu_live[b + 1] - l0;
@@ -616,6 +622,16 @@ int cache_plan(int num_layers, int mode_flags, const refcache_segments_t* seg, r
       add_rows(bt, tr, s0, ns, s0, ns, 0, 0);  // [ST; R] rows attend [ST; R] (R only when isolated)
     }
     add_rows(st, tr, l0, nl, l0, nl, c0, nc);  // live rows attend their own rows, then the cache
+    if (!f8) {
+      // in-slot build: the same rows and visibility, keys read from the slot
+      if (mode == REFCACHE_MASK_BEYOND_ALT) {  // the slot holds [ST; R]: key range A is the slot
+        add_rows(bs, tr, s0, na, c0, na, 0, 0);
+        add_rows(bs, tr, s0 + na, ns - na, c0, ns, 0, 0);
+      } else {  // anchors (range A, given apart), then R in the slot (range B)
+        add_rows(bs, tr, s0, ns, a0, na, c0, nc);
+      }
+    }
+    a0 += mode == REFCACHE_MASK_BEYOND_ALT ? 0 : na;
     if (nc > 0 && !f8) {
       CopySeg c{};
       c.src_row0 = mode == REFCACHE_MASK_BEYOND_ALT ? s0 : s0 + na;
@@ -626,12 +642,14 @@ int cache_plan(int num_layers, int mode_flags, const refcache_segments_t* seg, r
   }
   order_tasks(bt);
   order_tasks(st);
+  order_tasks(bs);
   const size_t slot_elems = static_cast<size_t>(cache_off[B]) * H * D;
   size_t off = 0;
   off = align_up(off + bt.size() * sizeof(Task), 256);
   off = align_up(off + st.size() * sizeof(Task), 256);
   off = align_up(off + cp.size() * sizeof(CopySeg), 256);
   off = align_up(off + qt.size() * sizeof(QuantTile), 256);
+  off = align_up(off + bs.size() * sizeof(Task), 256);
   const size_t layer_bytes = f8 ? fp8_layer_bytes(off8[B], H, D) : 2 * slot_elems * sizeof(__nv_bfloat16);
   const size_t total = off + static_cast<size_t>(num_layers) * layer_bytes;
   if (h) {
@@ -653,6 +671,8 @@ int cache_plan(int num_layers, int mode_flags, const refcache_segments_t* seg, r
     h->cache_rows = cache_off[B];
     h->slot_elems = static_cast<int64_t>(slot_elems);
     h->n_build = static_cast<int>(bt.size());
+    h->n_build_slot = static_cast<int>(bs.size());
+    h->anchor_rows = a0;
     h->n_step = static_cast<int>(st.size());
     h->n_copy = static_cast<int>(cp.size());
   }
@@ -660,6 +680,7 @@ int cache_plan(int num_layers, int mode_flags, const refcache_segments_t* seg, r
   if (step_tasks) *step_tasks = std::move(st);
   if (copies) *copies = std::move(cp);
   if (qtiles) *qtiles = std::move(qt);
+  if (slot_tasks) *slot_tasks = std::move(bs);
   *total_bytes = total;
   return REFCACHE_OK;
 }
@@ -744,7 +765,7 @@ extern "C" {
 
 size_t refcache_bytes(int num_layers, int mask_mode, const refcache_segments_t* seg) {
   size_t total = 0;
-  if (cache_plan(num_layers, mask_mode, seg, nullptr, nullptr, nullptr, nullptr, nullptr, &total) != 0) return 0;
+  if (cache_plan(num_layers, mask_mode, seg, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, &total) != 0) return 0;
   return total;
 }
 
@@ -752,11 +773,11 @@ int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refca
                     size_t dev_bytes) {
   if (!out) return fail(REFCACHE_ERR_INVALID_ARG, "out is NULL");
   refcache* h = new refcache();
-  std::vector<Task> bt, st;
+  std::vector<Task> bt, st, bs;
   std::vector<CopySeg> cp;
   std::vector<QuantTile> qt;
   size_t total = 0;
-  int rc = cache_plan(num_layers, mask_mode, seg, h, &bt, &st, &cp, &qt, &total);
+  int rc = cache_plan(num_layers, mask_mode, seg, h, &bt, &st, &cp, &qt, &bs, &total);
   if (rc) {
     delete h;
     return rc;
@@ -795,6 +816,8 @@ int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refca
   off = align_up(off + cp.size() * sizeof(CopySeg), 256);
   h->d_qtiles = reinterpret_cast<QuantTile*>(h->mem + off);
   off = align_up(off + qt.size() * sizeof(QuantTile), 256);
+  h->d_build_slot = reinterpret_cast<Task*>(h->mem + off);
+  off = align_up(off + bs.size() * sizeof(Task), 256);
   h->slots = reinterpret_cast<__nv_bfloat16*>(h->mem + off);
   h->slots8 = h->mem + off;
   cudaError_t e = cudaSuccess;
@@ -803,6 +826,8 @@ int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refca
   if (!cp.empty() && e == cudaSuccess) e = cudaMemcpy(h->d_copy, cp.data(), cp.size() * sizeof(CopySeg), cudaMemcpyHostToDevice);
   if (!qt.empty() && e == cudaSuccess)
     e = cudaMemcpy(h->d_qtiles, qt.data(), qt.size() * sizeof(QuantTile), cudaMemcpyHostToDevice);
+  if (!bs.empty() && e == cudaSuccess)
+    e = cudaMemcpy(h->d_build_slot, bs.data(), bs.size() * sizeof(Task), cudaMemcpyHostToDevice);
   if (e != cudaSuccess) {
     if (h->owns) cudaFree(h->mem);
     delete h;
@@ -858,7 +883,9 @@ int refcache_fp8_ptr(refcache_t* h, int layer, void** k8, void** vt8, void** sca
 
 int refcache_call_launches(refcache_t* h, int call) {
   if (!h) return fail(REFCACHE_ERR_INVALID_ARG, "cache is NULL");
-  if (call != 0 && call != 1) return fail(REFCACHE_ERR_INVALID_ARG, "call must be 0 (build) or 1 (step)");
+  if (call < 0 || call > 2)
+    return fail(REFCACHE_ERR_INVALID_ARG, "call must be 0 (build), 1 (step) or 2 (build in slot)");
+  if (call == 2) return h->f8 ? fail(REFCACHE_ERR_UNSUPPORTED, "an E4M3 cache has no in-slot build") : h->n_build_slot > 0;
   const int n_tasks = call == 0 ? h->n_build : h->n_step;
   const int cache_write = call == 0 && (h->n_copy > 0 || h->n_qtiles > 0) ? 1 : 0;
   if (n_tasks == 0) return cache_write;
@@ -907,6 +934,41 @@ int refcache_build(refcache_t* h, int layer, const void* q_static, const void* k
   Operands op{q_static, h->static_rows, k_static, v_static, h->static_rows, nullptr, nullptr, 0, o_static, lse_static};
   rc = run_attention(h->d_build, h->n_build, h->H, h->D, op, softmax_scale, info, s, nullptr, nullptr,
                      h->n_copy > 0 ? &cj : nullptr);
+  if (rc) return rc;
+  h->built[layer] = 1;
+  return REFCACHE_OK;
+}
+
+int refcache_build_in_slot(refcache_t* h, int layer, const void* q_static, const void* k_anchor,
+                           const void* v_anchor, void* o_static, float* lse_static, float softmax_scale, void* stream) {
+  int rc = check_handle_layer(h, layer);
+  if (rc) return rc;
+  if (h->f8)
+    return fail(REFCACHE_ERR_UNSUPPORTED, "refcache_build_in_slot needs a bf16 cache (an E4M3 cache is written by "
+                                          "refcache_build from the bf16 K and V)");
+  if ((rc = check_scale(softmax_scale)) != 0) return rc;
+  if ((rc = check_ptrs({q_static, o_static}, h->static_rows, "refcache_build_in_slot")) != 0) return rc;
+  const bool alt = h->mode == REFCACHE_MASK_BEYOND_ALT;
+  if (!alt && (rc = check_ptrs({k_anchor, v_anchor}, h->anchor_rows, "refcache_build_in_slot anchors")) != 0)
+    return rc;
+  DeviceInfo* info = nullptr;
+  if ((rc = enter_device(h, &info)) != 0) return rc;
+  void *kslot = nullptr, *vslot = nullptr;
+  refcache_kv_ptr(h, layer, &kslot, &vslot, nullptr);
+  const bool anchors = !alt && h->anchor_rows > 0;
+  const bool range_b = !alt && h->cache_rows > 0;
+  Operands op{q_static,
+              h->static_rows,
+              anchors ? k_anchor : kslot,
+              anchors ? v_anchor : vslot,
+              anchors ? h->anchor_rows : h->cache_rows,
+              range_b ? kslot : nullptr,
+              range_b ? vslot : nullptr,
+              range_b ? h->cache_rows : 0,
+              o_static,
+              lse_static};
+  rc = run_attention(h->d_build_slot, h->n_build_slot, h->H, h->D, op, softmax_scale, info,
+                     static_cast<cudaStream_t>(stream));
   if (rc) return rc;
   h->built[layer] = 1;
   return REFCACHE_OK;

@@ -30,7 +30,7 @@ EXPORTED = (
     "refcache_bytes", "refcache_create", "refcache_destroy", "refcache_kv_ptr", "refcache_layer_built",
     "refcache_build", "step_attention", "full_attention", "refcache_status", "refcache_set_wait_timeout_ns",
     "refcache_set_kernel", "refcache_debug_skip_first_load", "refcache_last_error", "refcache_version",
-    "full_attention_noalloc", "refcache_call_launches", "refcache_fp8_ptr",
+    "full_attention_noalloc", "refcache_call_launches", "refcache_fp8_ptr", "refcache_build_in_slot",
 )
 NOALLOC_MAX_TASKS = 16384
 
@@ -79,6 +79,7 @@ def load(path: Optional[str] = None):
     L.refcache_layer_built.argtypes = [vp, i32]
     L.refcache_call_launches.argtypes = [vp, i32]
     L.refcache_build.argtypes = [vp, i32, vp, vp, vp, vp, vp, f32, vp]
+    L.refcache_build_in_slot.argtypes = [vp, i32, vp, vp, vp, vp, vp, f32, vp]
     L.step_attention.argtypes = [vp, i32, vp, vp, vp, vp, vp, f32, vp]
     L.full_attention.argtypes = [i32, i32, i32, ctypes.POINTER(ctypes.c_int32), vp, vp, vp, vp, vp, f32, vp]
     L.full_attention_noalloc.argtypes = [i32, i32, i32, ctypes.POINTER(ctypes.c_int32), vp, vp, vp, vp, vp, f32,
@@ -273,8 +274,8 @@ class RefCache:
         return bool(r)
 
     def launches(self, call: str) -> int:
-        """Kernels one build ('build') or step ('step') call launches."""
-        r = load().refcache_call_launches(self.h, {"build": 0, "step": 1}[call])
+        """Kernels one build ('build'), step ('step') or in-slot build ('build_in_slot') call launches."""
+        r = load().refcache_call_launches(self.h, {"build": 0, "step": 1, "build_in_slot": 2}[call])
         _check(0 if r >= 0 else r)
         return int(r)
 
@@ -285,6 +286,24 @@ class RefCache:
         scale = default_scale(D) if scale is None else scale
         _check(load().refcache_build(self.h, layer, _ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), scale,
                                      _stream(stream)))
+
+    def build_in_slot(self, layer, q, k_anchor, v_anchor, o, lse=None, scale=None, stream=None):
+        """The prefill of a layer whose cached rows' K/V the caller already
+        wrote into the slots (``kv(layer)``); the anchors' K/V are passed apart
+        as [sum n_anchor, H, D] (None when there are none, or in the
+        alternative anchor reading, whose slots hold them)."""
+        H, D, n = self.seg.num_heads, self.seg.head_dim, self.seg.static_rows
+        for name, t in (("q", q), ("o", o)):
+            _check_thd(name, t, n, H, D)
+        n_a = sum(self.seg.n_anchor) if self.mask_mode != "beyond_alt" else 0
+        if n_a:
+            for name, t in (("k_anchor", k_anchor), ("v_anchor", v_anchor)):
+                _check_thd(name, t, n_a, H, D)
+        else:
+            k_anchor = v_anchor = None
+        scale = default_scale(D) if scale is None else scale
+        _check(load().refcache_build_in_slot(self.h, layer, _ptr(q), _ptr(k_anchor), _ptr(v_anchor), _ptr(o),
+                                             _ptr(lse), scale, _stream(stream)))
 
     def step(self, layer, q, k, v, o, lse=None, scale=None, stream=None):
         H, D, n = self.seg.num_heads, self.seg.head_dim, self.seg.live_rows
