@@ -3,7 +3,7 @@
  * plain C, without the Python binding.
  *
  *   test_abi cpu   sizing and argument checks; needs no device
- *   test_abi gpu   refcache_create / refcache_build / step_attention of a small
+ *   test_abi gpu   refcache_create / refcache_build (and refcache_build_in_slot) / step_attention of a small
  *                  ragged batch on the current GPU, head dims 64 and 128, both
  *                  outputs compared with the oracle's joint attention
  *                  (oracle/oracle.c, linked in) on the same input bytes
@@ -145,12 +145,44 @@ static int run_gpu_dim(int d) {
   CHECK(rc == REFCACHE_OK, "refcache_build %d", rc);
   rc = step_attention(h, 0, dev[4], dev[5], dev[6], dev[7], NULL, scale, NULL);
   CHECK(rc == REFCACHE_OK, "step_attention %d", rc);
+  /* the same prefill for a caller that writes the cached rows' K/V straight
+     into the slots (here by copying R's rows there) and passes the anchors apart */
+  refcache_t* h2 = NULL;
+  rc = refcache_create(&h2, 1, REFCACHE_MASK_BEYOND, &seg, NULL, 0);
+  CHECK(rc == REFCACHE_OK && h2, "refcache_create (in-slot) %d", rc);
+  void *kslot = NULL, *vslot = NULL, *da[2], *os2_d, *ol2_d;
+  int64_t crows = 0, na_tot = 0;
+  CHECK(refcache_kv_ptr(h2, 0, &kslot, &vslot, &crows) == REFCACHE_OK, "refcache_kv_ptr");
+  for (int b = 0; b < B; ++b) na_tot += reqs[b].n_st;
+  for (int i = 0; i < 2; ++i) CHECK(cudaMalloc(&da[i], na_tot ? (size_t)na_tot * row * 2 : 16) == cudaSuccess, "cudaMalloc");
+  CHECK(cudaMalloc(&os2_d, n_s * 2) == cudaSuccess && cudaMalloc(&ol2_d, n_l * 2) == cudaSuccess, "cudaMalloc");
+  int64_t c_rows = 0, a_rows = 0;
+  for (int b = 0; b < B; ++b) {
+    const size_t src_r = ((size_t)cu_static[b] + reqs[b].n_st) * row * 2, src_a = (size_t)cu_static[b] * row * 2;
+    const size_t nr = (size_t)reqs[b].n_r * row * 2, na = (size_t)reqs[b].n_st * row * 2;
+    CHECK(cudaMemcpy((char*)kslot + c_rows * row * 2, (char*)dev[1] + src_r, nr, cudaMemcpyDeviceToDevice) == cudaSuccess &&
+              cudaMemcpy((char*)vslot + c_rows * row * 2, (char*)dev[2] + src_r, nr, cudaMemcpyDeviceToDevice) == cudaSuccess &&
+              cudaMemcpy((char*)da[0] + a_rows * row * 2, (char*)dev[1] + src_a, na, cudaMemcpyDeviceToDevice) == cudaSuccess &&
+              cudaMemcpy((char*)da[1] + a_rows * row * 2, (char*)dev[2] + src_a, na, cudaMemcpyDeviceToDevice) == cudaSuccess,
+          "slot copy");
+    c_rows += reqs[b].n_r;
+    a_rows += reqs[b].n_st;
+  }
+  CHECK(c_rows == crows, "slot rows %lld, expected %lld", (long long)crows, (long long)c_rows);
+  rc = refcache_build_in_slot(h2, 0, dev[0], da[0], da[1], os2_d, NULL, scale, NULL);
+  CHECK(rc == REFCACHE_OK, "refcache_build_in_slot %d", rc);
+  rc = step_attention(h2, 0, dev[4], dev[5], dev[6], ol2_d, NULL, scale, NULL);
+  CHECK(rc == REFCACHE_OK, "step_attention (in-slot cache) %d", rc);
   rc = refcache_status(NULL);
   CHECK(rc == REFCACHE_OK, "refcache_status %d", rc);
   uint16_t* os = (uint16_t*)malloc(n_s * 2 + 2);
   uint16_t* ol = (uint16_t*)malloc(n_l * 2 + 2);
+  uint16_t* os2 = (uint16_t*)malloc(n_s * 2 + 2);
+  uint16_t* ol2 = (uint16_t*)malloc(n_l * 2 + 2);
   CHECK(cudaMemcpy(os, dev[3], n_s * 2, cudaMemcpyDeviceToHost) == cudaSuccess, "copy out");
   CHECK(cudaMemcpy(ol, dev[7], n_l * 2, cudaMemcpyDeviceToHost) == cudaSuccess, "copy out");
+  CHECK(cudaMemcpy(os2, os2_d, n_s * 2, cudaMemcpyDeviceToHost) == cudaSuccess, "copy out");
+  CHECK(cudaMemcpy(ol2, ol2_d, n_l * 2, cudaMemcpyDeviceToHost) == cudaSuccess, "copy out");
   double worst = 0;
   for (int b = 0; b < B; ++b) {
     const req_t r = reqs[b];
@@ -174,6 +206,12 @@ static int run_gpu_dim(int d) {
     const double mx_s = compare(os + (size_t)cu_static[b] * row, out + (size_t)n_live * row, (size_t)n_stat * row, &mean_s);
     CHECK(mx_l <= 2e-2 && mean_l <= 2e-3, "d=%d request %d step: max %.3e mean %.3e", d, b, mx_l, mean_l);
     CHECK(mx_s <= 2e-2 && mean_s <= 2e-3, "d=%d request %d prefill: max %.3e mean %.3e", d, b, mx_s, mean_s);
+    double mean_l2, mean_s2;
+    const double mx_l2 = compare(ol2 + (size_t)cu_live[b] * row, out, (size_t)n_live * row, &mean_l2);
+    const double mx_s2 = compare(os2 + (size_t)cu_static[b] * row, out + (size_t)n_live * row, (size_t)n_stat * row, &mean_s2);
+    CHECK(mx_l2 <= 2e-2 && mean_l2 <= 2e-3, "d=%d request %d step (in-slot cache): max %.3e", d, b, mx_l2);
+    CHECK(mx_s2 <= 2e-2 && mean_s2 <= 2e-3, "d=%d request %d in-slot prefill: max %.3e", d, b, mx_s2);
+    if (mx_s2 > worst) worst = mx_s2;
     if (mx_l > worst) worst = mx_l;
     if (mx_s > worst) worst = mx_s;
     free(q);
@@ -182,8 +220,13 @@ static int run_gpu_dim(int d) {
     free(out);
   }
   refcache_destroy(h);
+  refcache_destroy(h2);
   for (int i = 0; i < 8; ++i) cudaFree(dev[i]);
-  free(qs); free(ks); free(vs); free(ql); free(kl); free(vl); free(os); free(ol);
+  cudaFree(da[0]);
+  cudaFree(da[1]);
+  cudaFree(os2_d);
+  cudaFree(ol2_d);
+  free(qs); free(ks); free(vs); free(ql); free(kl); free(vl); free(os); free(ol); free(os2); free(ol2);
   printf("gpu d=%d ok (max abs %.3e)\n", d, worst);
   return 0;
 }
