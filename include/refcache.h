@@ -161,12 +161,13 @@ REFCACHE_API size_t refcache_bytes(int num_layers, int mask_mode, const refcache
  * the caller, not freed).  Synchronous.  *out is set only on success.
  *
  * For head_dim 128 it also plans, for the current device, the per-item work
- * list of the step: when its (query tile, head) items do not fill the last
- * round of the GPU's CTA pairs evenly, the items of that round are split by
- * key range into 2-8 parts whose outputs a combine kernel merges.  This list
- * and an fp32 workspace for the parts (parts x 256 rows x (head_dim + 1) x 4
- * bytes, e.g. 27 MB at 1024^2 with five references) are one more cudaMalloc,
- * freed by refcache_destroy.  Which step items are split depends on the whole
+ * lists of the prefill and the step, each (query tile, head) item assigned to
+ * the CTA pair with the least work so far (longest first).  When the step's
+ * items do not fill the last round of the GPU's CTA pairs evenly, the items of
+ * that round are split by key range into 2-8 parts whose outputs a combine
+ * kernel merges.  These lists and an fp32 workspace for the parts (parts x 256
+ * rows x (head_dim + 1) x 4 bytes, e.g. 27 MB at 1024^2 with five references)
+ * are one more cudaMalloc, freed by refcache_destroy.  Which step items are split depends on the whole
  * batch and the device, so a step output's last bits may differ between
  * batches (never by more than the rounding of a split).  The prefill is never
  * split: refcache_build's outputs and cache bytes for a request depend only on

@@ -14,7 +14,9 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <functional>
 #include <mutex>
+#include <queue>
 #include <string>
 #include <vector>
 
@@ -498,6 +500,42 @@ void plan_items(const std::vector<Task>& tasks, int H, int clusters, int tile, s
   items->insert(items->end(), parts.begin(), parts.end());
 }
 
+// Lays a per-item list (longest items first) out for a persistent grid of
+// `clusters` CTA pairs, pair c taking slots c, c + clusters, c + 2 clusters,
+// ...: each item goes to the pair with the least work so far (longest
+// processing time first, ties to the lower pair), in the list's order, and
+// slots a pair does not need are empty tasks (no rows, no keys).  Work = MMA
+// groups: key tiles + 2.  Only the order changes, not any item's arithmetic.
+std::vector<Task> lpt_layout(const std::vector<Task>& items, int clusters, int tile) {
+  const int n = static_cast<int>(items.size());
+  const int c = std::min(n, clusters);
+  if (c <= 1) return items;
+  std::vector<int> order(n);
+  for (int i = 0; i < n; ++i) order[i] = i;
+  auto groups = [&](const Task& t) -> int64_t {
+    const int64_t nkv = (t.a_len + tile - 1) / tile + (t.b_len + tile - 1) / tile;
+    return nkv > 0 ? nkv + 2 : 0;
+  };
+  std::stable_sort(order.begin(), order.end(),
+                   [&](int x, int y) { return groups(items[x]) > groups(items[y]); });
+  using Load = std::pair<int64_t, int>;
+  std::priority_queue<Load, std::vector<Load>, std::greater<Load>> pq;
+  for (int i = 0; i < c; ++i) pq.push({0, i});
+  std::vector<std::vector<int>> per(c);
+  for (int i : order) {
+    const Load l = pq.top();
+    pq.pop();
+    per[l.second].push_back(i);
+    pq.push({l.first + groups(items[i]), l.second});
+  }
+  size_t depth = 0;
+  for (const auto& v : per) depth = std::max(depth, v.size());
+  std::vector<Task> out(static_cast<size_t>(c) * depth, Task{});
+  for (int p = 0; p < c; ++p)
+    for (size_t k = 0; k < per[p].size(); ++k) out[p + k * c] = items[per[p][k]];
+  return out;
+}
+
 // Work list of full_attention_noalloc: a fixed array in static device memory
 // (no allocation at call time), shared by every call on a device.
 __device__ __align__(256) static Task g_noalloc_tasks[REFCACHE_NOALLOC_MAX_TASKS];
@@ -534,10 +572,11 @@ struct refcache {
   int n_step = 0;
   CopySeg* d_copy = nullptr;
   int n_copy = 0;
-  // per-item list of the head-dim-128 step with split items, in a separate
-  // allocation: [step items | step jobs | part_o | part_lse]
+  // per-item lists of the head-dim-128 kernel, laid out for the persistent
+  // grid (the step's with split items), in a separate allocation:
+  // [build items | step items | step jobs | part_o | part_lse]
   uint8_t* aux = nullptr;
-  ItemList step_items;
+  ItemList build_items, step_items;
   __nv_bfloat16* slots = nullptr;
   int64_t slot_elems = 0;
   // E4M3 cache (REFCACHE_CACHE_FP8): per layer [k8 | vt8 | scales] of
@@ -701,27 +740,41 @@ int check_ptrs(std::initializer_list<const void*> ps, int64_t rows, const char* 
   return REFCACHE_OK;
 }
 
-// Per-item list of the step of a head-dim-128 handle, with the last round of
-// items split, in one allocation of its own (the caller-sized cache memory is
-// not touched).  The prefill is never split: each of its items runs whole on
-// one CTA pair, so a request's prefill outputs depend on its own (N_ST, N_R)
-// only -- not on the other requests of the batch, nor on the device's SM count
-// -- and the cached block is reproduced bit for bit (Sec. 3.3).
-int plan_split_items(refcache* h, DeviceInfo* info, const std::vector<Task>& st) {
+// Per-item lists of a head-dim-128 handle for the current device, in one
+// allocation of their own (the caller-sized cache memory is not touched):
+// the step's, with the last round of items split, and the prefill's, whose
+// items are never split: each runs whole on one CTA pair, so a request's
+// prefill outputs depend on its own (N_ST, N_R) only -- not on the other
+// requests of the batch, nor on the device's SM count -- and the cached block
+// is reproduced bit for bit (Sec. 3.3).  Both are laid out by lpt_layout.
+int plan_split_items(refcache* h, DeviceInfo* info, const std::vector<Task>& bt, const std::vector<Task>& st) {
   // planned for the step kernel selected now (key tiles of tc2_tile(); the
-  // parts stay correct, only less even, if another tile size runs them)
+  // parts and the layout stay correct, only less even, if another tile size
+  // or grid runs them)
   const bool f8 = h->f8 && h->rows_pad > 0;
-  const int tile = tc2_tile(f8);
-  int clusters = 0;
+  const int tile = tc2_tile(f8), tile_b = tc2_tile(false);
+  int clusters = 0, clusters_b = 0;
   int rc = f8 ? tc2_clusters<true, 128>(info, &clusters)
               : tile == 128 ? tc2_clusters<false, 128>(info, &clusters) : tc2_clusters<false, 192>(info, &clusters);
   if (rc) return rc;
-  std::vector<Task> si;
+  rc = tile_b == 128 ? tc2_clusters<false, 128>(info, &clusters_b) : tc2_clusters<false, 192>(info, &clusters_b);
+  if (rc) return rc;
+  std::vector<Task> si, bi;
   std::vector<CombineJob> sj;
   int parts = 0;
   plan_items(st, h->H, clusters, tile, &si, &sj, &parts);
+  si = lpt_layout(si, clusters, tile);
+  for (int hd = 0; hd < h->H; ++hd)
+    for (Task t : bt) {
+      t.head = hd;
+      t.part = 0;
+      bi.push_back(t);
+    }
+  bi = lpt_layout(bi, clusters_b, tile_b);
   const int rows = task_rows(h->D);
   size_t off = 0;
+  const size_t o_bi = off;
+  off = align_up(off + bi.size() * sizeof(Task), 256);
   const size_t o_si = off;
   off = align_up(off + si.size() * sizeof(Task), 256);
   const size_t o_sj = off;
@@ -738,12 +791,15 @@ int plan_split_items(refcache* h, DeviceInfo* info, const std::vector<Task>& st)
   auto put = [&](size_t o, const void* src, size_t n) -> cudaError_t {
     return n ? cudaMemcpy(h->aux + o, src, n, cudaMemcpyHostToDevice) : cudaSuccess;
   };
-  if ((e = put(o_si, si.data(), si.size() * sizeof(Task))) != cudaSuccess ||
+  if ((e = put(o_bi, bi.data(), bi.size() * sizeof(Task))) != cudaSuccess ||
+      (e = put(o_si, si.data(), si.size() * sizeof(Task))) != cudaSuccess ||
       (e = put(o_sj, sj.data(), sj.size() * sizeof(CombineJob))) != cudaSuccess) {
     cudaFree(h->aux);
     h->aux = nullptr;
     return cuda_fail(e, "cudaMemcpy(split work list)");
   }
+  h->build_items = ItemList{reinterpret_cast<Task*>(h->aux + o_bi), static_cast<int>(bi.size()), nullptr, 0,
+                            nullptr, nullptr};
   h->step_items = ItemList{reinterpret_cast<Task*>(h->aux + o_si), static_cast<int>(si.size()),
                            reinterpret_cast<CombineJob*>(h->aux + o_sj), static_cast<int>(sj.size()),
                            reinterpret_cast<float*>(h->aux + o_po), reinterpret_cast<float*>(h->aux + o_pl)};
@@ -833,7 +889,7 @@ int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refca
     delete h;
     return cuda_fail(e, "cudaMemcpy(work tables)");
   }
-  if (h->D == 128 && (rc = plan_split_items(h, info, st)) != 0) {
+  if (h->D == 128 && (rc = plan_split_items(h, info, bt, st)) != 0) {
     if (h->owns) cudaFree(h->mem);
     delete h;
     return rc;
@@ -932,8 +988,8 @@ int refcache_build(refcache_t* h, int layer, const void* q_static, const void* k
     cj.rows = h->cache_rows;
   }
   Operands op{q_static, h->static_rows, k_static, v_static, h->static_rows, nullptr, nullptr, 0, o_static, lse_static};
-  rc = run_attention(h->d_build, h->n_build, h->H, h->D, op, softmax_scale, info, s, nullptr, nullptr,
-                     h->n_copy > 0 ? &cj : nullptr);
+  rc = run_attention(h->d_build, h->n_build, h->H, h->D, op, softmax_scale, info, s,
+                     h->build_items.items ? &h->build_items : nullptr, nullptr, h->n_copy > 0 ? &cj : nullptr);
   if (rc) return rc;
   h->built[layer] = 1;
   return REFCACHE_OK;
