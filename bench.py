@@ -360,6 +360,7 @@ def run_ours(args, ws, rank, local):
             "sustained_note": "the sustained peak was measured at a power-capped median SM clock of about "
                               "1.4 GHz; this kernel's timed region runs near 2 GHz, so it is context only",
             "nominal_at_clock": nominal_at_clock(achieved, clocks.get("sm_mhz"), sms, peak_mult),
+            "exp_floor": exp_floor(acc.step_units(w.requests) * H, t_step, clocks.get("sm_mhz"), sms),
             "traffic": recorded_traffic(w.name, args.kernel) if args.cache == "bf16" else None,
             "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum, one step_attention launch"
                               " (profiles/); null when the kernel sources changed since",
@@ -389,6 +390,22 @@ def nominal_at_clock(achieved, sm_mhz, sms, mult=1.0):
     ceiling = mult * 8192.0 * sms * sm_mhz * 1e6 / 1e12
     return {"sm_mhz": sm_mhz, "sms": sms, "flop_per_clk_per_sm": mult * 8192, "tflops": ceiling,
             "frac": achieved / ceiling}
+
+
+# Exponentials per clock per SM of ex2.approx.f32 (MUFU), measured on this
+# GPU by a probe kernel: one warp instruction per 4 cycles per sub-partition.
+MUFU_EX2_PER_CLK_PER_SM = 32
+
+
+def exp_floor(units, secs, sm_mhz, sms):
+    """The secondary ALU limit: one exponential per visible (query, key) pair
+    of one head against the MUFU rate at the sampled clock."""
+    if not sm_mhz:
+        return None
+    floor = units / (MUFU_EX2_PER_CLK_PER_SM * sms * sm_mhz * 1e6)
+    return {"exps": units, "ex2_per_clk_per_sm": MUFU_EX2_PER_CLK_PER_SM, "sm_mhz": sm_mhz,
+            "floor_ms": floor * 1e3, "frac_of_step": floor / secs,
+            "note": "MUFU time the exponentials need at the sampled clock, as a share of the step"}
 
 
 def gpu_randn_bf16(shape, seed: int, dev):

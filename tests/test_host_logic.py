@@ -43,3 +43,19 @@ def test_workload_shapes():
     assert w.cu_live[-1] == sum(r.n_lt + r.n_x for r in w.requests)
     q, k, v = workloads.static_qkv(workloads.TINY)
     assert q.shape == (288, 4, 64)
+
+
+def test_bench_clock_ceilings():
+    """The bench line's two clock-based figures: the tensor pipe's ceiling
+    (8192 dense bf16 FLOPs per clock per SM) and the exponential floor (one
+    MUFU ex2 per visible pair, 32 per clock per SM), at a given clock."""
+    import bench
+
+    n = bench.nominal_at_clock(1000.0, 2000.0, 152)
+    assert n["tflops"] == pytest.approx(8192 * 152 * 2.0e9 / 1e12) and n["frac"] == pytest.approx(1000.0 / n["tflops"])
+    assert bench.nominal_at_clock(1000.0, None, 152) is None
+    w = workloads.EDIT_1024_5REF
+    exps = acc.step_units(w.requests) * w.num_heads
+    f = bench.exp_floor(exps, 1e-3, 2000.0, 152)
+    assert f["floor_ms"] == pytest.approx(exps / (32 * 152 * 2.0e9) * 1e3)
+    assert f["frac_of_step"] == pytest.approx(f["floor_ms"] / 1.0)
