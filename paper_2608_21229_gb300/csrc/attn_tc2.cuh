@@ -3,20 +3,27 @@
 // two CTAs on neighbouring SMs (tcgen05 cta_group::2, M = 256).
 //
 // Why pairs: with one 128-row query tile per SM, each S/P.V pair of MMAs
-// (1024 tensor cycles) needs a fresh 32 KB K tile and 32 KB V tile in that
-// SM's shared memory.  The tensor core's operand reads (about 96 KB per pair)
-// plus those 64 KB of TMA fills exceed what one SM's shared memory delivers
-// in 1024 cycles (128 bytes per cycle), so the tensor core waits for data.  A
-// CTA pair shares every K/V tile: CTA r holds keys [64 r, 64 r + 64) of each
-// K tile and head-dim columns [64 r, 64 r + 64) of each V tile (the B operand
-// of a cta_group::2 MMA is split along N between the two CTAs), while each
-// CTA keeps its own 128 query rows (A is split along M).  Per SM this halves
-// the tile bytes fetched and the B-operand bytes read, for the same MMA work.
+// (1024 tensor cycles at 128-key tiles) needs a fresh 32 KB K tile and 32 KB
+// V tile in that SM's shared memory.  The tensor core's operand reads (about
+// 96 KB per pair) plus those 64 KB of TMA fills exceed what one SM's shared
+// memory delivers in 1024 cycles (128 bytes per cycle), so the tensor core
+// waits for data.  A CTA pair shares every K/V tile: CTA r holds keys
+// [kBN/2 r, kBN/2 (r + 1)) of each K tile and head-dim columns [64 r, 64 r +
+// 64) of each V tile (the B operand of a cta_group::2 MMA is split along N
+// between the two CTAs), while each CTA keeps its own 128 query rows (A is
+// split along M).  Per SM this halves the tile bytes fetched and the
+// B-operand bytes read, for the same MMA work.
+//
+// Key tiles (kBN): 192 keys for the bf16 cache, 128 for the E4M3 cache and
+// the 128-key comparison variant.  At 192 keys P is written over the first
+// half of its own S buffer, which is what makes two 192-column S buffers and
+// the 128-column O fit in the 512 TMEM columns; each handshake then carries
+// 1536 tensor cycles of MMAs instead of 1024 (see Cfg).
 //
 // Cluster of 2 CTAs (rank 0 = leader), 224 threads each (352 in the E4M3
 // kernel, whose 8 softmax warps split each row's columns, see below):
 //   warps 0-3  softmax: thread l of warp w owns row 32 w + l of this CTA's
-//              128 rows (its TMEM lane), all 128 score columns of a tile
+//              128 rows (its TMEM lane), all kBN score columns of a tile
 //   warp 4     TMA producer: this CTA's Q rows and its halves of the K and V
 //              tiles; completion is counted on the leader's barriers
 //   warp 5     both CTAs: TMEM allocation (a pair operation); leader only:
@@ -27,17 +34,20 @@
 // One softmax warp per SM sub-partition leaves the MMA warp's sub-partition
 // with a single busy warp beside it, and a row needs no partner thread.
 // An item is a task of up to 256 query rows: CTA r takes rows
-// [128 r, 128 r + 128).  Items are taken cluster by cluster, head-major.
+// [128 r, 128 r + 128).  Items are taken cluster by cluster from a per-item
+// list laid out on the host, or head-major from the task list.
 //
 // Work is done item by item (an item = a task of up to 256 rows x one
 // head).  An item with n key tiles is a sequence of n + 2 MMA groups:
 //   group G + 0, G + 1     S_0 = Q K_0^T, S_1 = Q K_1^T (the second is empty
 //                          when n = 1)
-//   group G + 2 + j        O += P_j V_j, interleaved MMA by MMA with
-//                          S_j+2 = Q K_j+2^T when j + 2 < n
+//   group G + 2 + j        O += P_j V_j with S_j+2 = Q K_j+2^T when j + 2 < n
+//                          (all P.V MMAs first when S_j+2 overwrites P_j,
+//                          else interleaved MMA by MMA)
 // numbered g = 0, 1, 2, ... over all items of the cluster.  Group g reads
-// ring stage g % 4 (K of its S, V of its P.V; 32 KB per CTA).  Tiles are also
-// numbered over all items (t); S_t and P_t live in TMEM buffer t % 2.
+// ring stage g % kStages (K of its S, V of its P.V; 48 KB per CTA at 192-key
+// tiles, 32 KB at 128).  Tiles are also numbered over all items (t); S_t and
+// P_t live in TMEM buffer t % 2.
 //
 // Synchronisation is built so that the MMA thread does as little as possible
 // between its MMAs: a tcgen05.mma blocks its thread until the tensor core
