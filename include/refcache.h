@@ -310,13 +310,23 @@ REFCACHE_API int full_attention_noalloc(int batch, int num_heads, int head_dim, 
  * Synchronise `stream`, then read and clear the current device's error word
  * written by kernels whose bounded waits ran out.  Returns REFCACHE_OK,
  * REFCACHE_ERR_TIMEOUT or REFCACHE_ERR_CUDA.
- * The word is one per device, not one per cache: every kernel of this library
- * on the device (any cache, any stream, full_attention too) writes the same
- * word, and the first refcache_status call that reads it clears it.  With
- * several caches in flight on one device a timeout therefore says that some
- * launch on the device gave up, not which cache's.
+ * The word is one per device: every kernel of this library on the device (any
+ * cache, any stream, full_attention too) writes it, and the first
+ * refcache_status call that reads it clears it.  To learn which cache's launch
+ * gave up, use refcache_cache_status.
  */
 REFCACHE_API int refcache_status(void* stream);
+
+/*
+ * The same for one cache: synchronise `stream`, then read and clear the error
+ * word of `cache`, which the kernels launched by refcache_build,
+ * refcache_build_in_slot and step_attention on this cache set (besides the
+ * device word) when a bounded wait runs out.  Returns REFCACHE_OK,
+ * REFCACHE_ERR_TIMEOUT, REFCACHE_ERR_INVALID_ARG (NULL cache, or the current
+ * device is not the cache's) or REFCACHE_ERR_CUDA.  It clears only this
+ * cache's word, and refcache_status only the device word.
+ */
+REFCACHE_API int refcache_cache_status(refcache_t* cache, void* stream);
 
 /* Wait limit of every in-kernel wait, nanoseconds (default 1e9).  Returns the old value. */
 REFCACHE_API uint64_t refcache_set_wait_timeout_ns(uint64_t ns);

@@ -85,7 +85,14 @@ struct Smem {
 struct Ctl {
   volatile int* abort_flag;
   uint64_t timeout_ns;
+  int* status;  // the launching cache's own error word, or null
 };
+
+// A bounded wait ran out at `where`: the device word, and the cache's own.
+__device__ __forceinline__ void report_timeout(int* status, int where) {
+  atomicCAS(&g_rc_status, 0, RC_DEV_TIMEOUT_BASE + where);
+  if (status) atomicCAS(status, 0, RC_DEV_TIMEOUT_BASE + where);
+}
 
 // Bounded wait on one mbarrier phase by one thread.
 __device__ __forceinline__ bool wait_one(uint32_t bar, uint32_t parity, const Ctl& c, int where) {
@@ -97,7 +104,7 @@ __device__ __forceinline__ bool wait_one(uint32_t bar, uint32_t parity, const Ct
     if (*c.abort_flag) return false;
     if (globaltimer_ns() - t0 > c.timeout_ns) {
       *c.abort_flag = 1;
-      atomicCAS(&g_rc_status, 0, RC_DEV_TIMEOUT_BASE + where);
+      report_timeout(c.status, where);
       return false;
     }
   }
@@ -214,7 +221,7 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   if (base - raw + L::kUsed > L::kDynamic) {  // the allocation cannot hold the aligned layout
-    if (threadIdx.x == 0) atomicCAS(&g_rc_status, 0, RC_DEV_TIMEOUT_BASE + 99);
+    if (threadIdx.x == 0) report_timeout(args.status, 99);
     return;
   }
 
@@ -244,7 +251,7 @@ __global__ void __launch_bounds__(tc::kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_holder;
-  const Ctl ctl{abort_flag, args.timeout_ns};
+  const Ctl ctl{abort_flag, args.timeout_ns, args.status};
 
   if (warp == 8) {
     // ------------------------------------------------------------ producer

@@ -204,7 +204,7 @@ __device__ __forceinline__ bool wait_cl(uint32_t bar, uint32_t parity, const Ctl
     if (*c.abort_flag) return false;
     if (globaltimer_ns() - t0 > c.timeout_ns) {
       *c.abort_flag = 1;
-      atomicCAS(&g_rc_status, 0, RC_DEV_TIMEOUT_BASE + where);
+      tc::report_timeout(c.status, where);
       return false;
     }
   }
@@ -259,7 +259,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
   const int n_clusters = static_cast<int>(gridDim.x >> 1);
   // Both CTAs of a pair get the same layout, so both leave here together.
   if (base - raw + L::kUsed > L::kDynamic) {
-    if (threadIdx.x == 0) atomicCAS(&g_rc_status, 0, RC_DEV_TIMEOUT_BASE + 99);
+    if (threadIdx.x == 0) tc::report_timeout(args.status, 99);
     return;
   }
 
@@ -296,7 +296,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
   grid_dependency_wait();
   if (threadIdx.x == 0) grid_launch_dependents();
   const uint32_t tmem = *tmem_holder;
-  const Ctl ctl{abort_flag, args.timeout_ns};
+  const Ctl ctl{abort_flag, args.timeout_ns, args.status};
   auto lbar = [&](int i) -> uint32_t { return mapa_shared(bar(i), 0); };  // leader's barrier i
 
   if (warp == Cfg::kProducerWarp) {

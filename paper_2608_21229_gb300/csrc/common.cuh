@@ -56,6 +56,7 @@ struct AttnArgs {
   const __nv_bfloat16* va;
   const __nv_bfloat16* kb;
   const __nv_bfloat16* vb;
+  int* status;  // the launching cache's own error word (null: the device word only)
 };
 
 // One item whose key range was split into parts: the combine kernel merges
@@ -67,7 +68,9 @@ struct CombineJob {
 static_assert(sizeof(CombineJob) == 32, "CombineJob layout is part of the device work list");
 
 // Device error word (one per device that loads the library); kernels set it
-// when a bounded wait runs out, refcache_status() reads and clears it.
+// when a bounded wait runs out, refcache_status() reads and clears it.  A
+// launch made for a cache also sets that cache's own word (AttnArgs::status),
+// which refcache_cache_status() reads and clears.
 #define RC_DEV_TIMEOUT_BASE 0x1000
 __device__ int g_rc_status;
 

@@ -297,6 +297,7 @@ struct Operands {
   int64_t b_rows;
   void* o;
   float* lse;
+  int* status = nullptr;  // the cache's own error word, if the launch is for a cache
 };
 
 // Key range B as an E4M3 cache (cache_fp8.cuh): codes of K [rows_pad, H, 128],
@@ -370,6 +371,7 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
   a.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634074);
   a.rows_per_task = task_rows(D);
   a.timeout_ns = g_timeout_ns.load();
+  a.status = op.status;
   a.q = static_cast<const __nv_bfloat16*>(op.q);
   a.ka = static_cast<const __nv_bfloat16*>(op.ka);
   a.va = static_cast<const __nv_bfloat16*>(op.va);
@@ -568,6 +570,7 @@ struct refcache {
   Task* d_build_slot = nullptr;
   int n_build_slot = 0;
   int64_t anchor_rows = 0;
+  int* d_status = nullptr;  // this cache's error word (device int), see refcache_cache_status
   Task* d_step = nullptr;
   int n_step = 0;
   CopySeg* d_copy = nullptr;
@@ -689,6 +692,7 @@ int cache_plan(int num_layers, int mode_flags, const refcache_segments_t* seg, r
   off = align_up(off + cp.size() * sizeof(CopySeg), 256);
   off = align_up(off + qt.size() * sizeof(QuantTile), 256);
   off = align_up(off + bs.size() * sizeof(Task), 256);
+  off = align_up(off + sizeof(int), 256);  // the cache's error word
   const size_t layer_bytes = f8 ? fp8_layer_bytes(off8[B], H, D) : 2 * slot_elems * sizeof(__nv_bfloat16);
   const size_t total = off + static_cast<size_t>(num_layers) * layer_bytes;
   if (h) {
@@ -874,6 +878,8 @@ int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refca
   off = align_up(off + qt.size() * sizeof(QuantTile), 256);
   h->d_build_slot = reinterpret_cast<Task*>(h->mem + off);
   off = align_up(off + bs.size() * sizeof(Task), 256);
+  h->d_status = reinterpret_cast<int*>(h->mem + off);
+  off = align_up(off + sizeof(int), 256);
   h->slots = reinterpret_cast<__nv_bfloat16*>(h->mem + off);
   h->slots8 = h->mem + off;
   cudaError_t e = cudaSuccess;
@@ -884,6 +890,7 @@ int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refca
     e = cudaMemcpy(h->d_qtiles, qt.data(), qt.size() * sizeof(QuantTile), cudaMemcpyHostToDevice);
   if (!bs.empty() && e == cudaSuccess)
     e = cudaMemcpy(h->d_build_slot, bs.data(), bs.size() * sizeof(Task), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemset(h->d_status, 0, sizeof(int));
   if (e != cudaSuccess) {
     if (h->owns) cudaFree(h->mem);
     delete h;
@@ -987,7 +994,8 @@ int refcache_build(refcache_t* h, int layer, const void* q_static, const void* k
     cj.row_u4 = h->H * h->D * 2 / 16;
     cj.rows = h->cache_rows;
   }
-  Operands op{q_static, h->static_rows, k_static, v_static, h->static_rows, nullptr, nullptr, 0, o_static, lse_static};
+  Operands op{q_static, h->static_rows, k_static, v_static, h->static_rows, nullptr, nullptr, 0, o_static, lse_static,
+              h->d_status};
   rc = run_attention(h->d_build, h->n_build, h->H, h->D, op, softmax_scale, info, s,
                      h->build_items.items ? &h->build_items : nullptr, nullptr, h->n_copy > 0 ? &cj : nullptr);
   if (rc) return rc;
@@ -1022,7 +1030,8 @@ int refcache_build_in_slot(refcache_t* h, int layer, const void* q_static, const
               range_b ? vslot : nullptr,
               range_b ? h->cache_rows : 0,
               o_static,
-              lse_static};
+              lse_static,
+              h->d_status};
   rc = run_attention(h->d_build_slot, h->n_build_slot, h->H, h->D, op, softmax_scale, info,
                      static_cast<cudaStream_t>(stream));
   if (rc) return rc;
@@ -1050,7 +1059,8 @@ int step_attention(refcache_t* h, int layer, const void* q_live, const void* k_l
   } else if (!h->f8) {
     refcache_kv_ptr(h, layer, &kslot, &vslot, nullptr);
   }
-  Operands op{q_live, h->live_rows, k_live, v_live, h->live_rows, kslot, vslot, h->cache_rows, o_live, lse_live};
+  Operands op{q_live, h->live_rows, k_live, v_live, h->live_rows, kslot, vslot, h->cache_rows, o_live, lse_live,
+              h->d_status};
   return run_attention(h->d_step, h->n_step, h->H, h->D, op, softmax_scale, info, static_cast<cudaStream_t>(stream),
                        h->step_items.items ? &h->step_items : nullptr, use_f8 ? &f8 : nullptr);
 }
@@ -1168,6 +1178,25 @@ int refcache_status(void* stream) {
     e = cudaMemcpyToSymbol(rc::g_rc_status, &zero, sizeof(int));
     if (e != cudaSuccess) return cuda_fail(e, "clear device error word");
     return fail(REFCACHE_ERR_TIMEOUT, "a kernel wait ran out (site %d)", v - RC_DEV_TIMEOUT_BASE);
+  }
+  return REFCACHE_OK;
+}
+
+int refcache_cache_status(refcache_t* h, void* stream) {
+  if (!h) return fail(REFCACHE_ERR_INVALID_ARG, "cache is NULL");
+  DeviceInfo* info = nullptr;
+  int rc = enter_device(h, &info);
+  if (rc) return rc;
+  cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+  int v = 0;
+  e = cudaMemcpy(&v, h->d_status, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "read the cache's error word");
+  if (v != 0) {
+    e = cudaMemset(h->d_status, 0, sizeof(int));
+    if (e != cudaSuccess) return cuda_fail(e, "clear the cache's error word");
+    return fail(REFCACHE_ERR_TIMEOUT, "a kernel wait of a launch for this cache ran out (site %d)",
+                v - RC_DEV_TIMEOUT_BASE);
   }
   return REFCACHE_OK;
 }

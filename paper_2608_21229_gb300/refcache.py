@@ -31,6 +31,7 @@ EXPORTED = (
     "refcache_build", "step_attention", "full_attention", "refcache_status", "refcache_set_wait_timeout_ns",
     "refcache_set_kernel", "refcache_debug_skip_first_load", "refcache_last_error", "refcache_version",
     "full_attention_noalloc", "refcache_call_launches", "refcache_fp8_ptr", "refcache_build_in_slot",
+    "refcache_cache_status",
 )
 NOALLOC_MAX_TASKS = 16384
 
@@ -85,6 +86,7 @@ def load(path: Optional[str] = None):
     L.full_attention_noalloc.argtypes = [i32, i32, i32, ctypes.POINTER(ctypes.c_int32), vp, vp, vp, vp, vp, f32,
                                          vp]
     L.refcache_status.argtypes = [vp]
+    L.refcache_cache_status.argtypes = [vp, vp]
     L.refcache_set_wait_timeout_ns.argtypes = [ctypes.c_uint64]
     L.refcache_set_wait_timeout_ns.restype = ctypes.c_uint64
     L.refcache_set_kernel.argtypes = [i32]
@@ -267,6 +269,11 @@ class RefCache:
 
         return (view(k, n * H * D).view(n, H, D), view(v, n * H * D).view(H, D, n),
                 view(sc, (n // 128) * H * 16).view(torch.float32).view(n // 128, H, 4))
+
+    def status(self, stream=None) -> int:
+        """Synchronise the stream and return (and clear) this cache's own error
+        word as a status code: a bounded wait of one of its launches ran out."""
+        return int(load().refcache_cache_status(self.h, _stream(stream)))
 
     def built(self, layer: int) -> bool:
         r = load().refcache_layer_built(self.h, layer)

@@ -3,9 +3,10 @@
 Every wait inside the tcgen05 kernel is bounded.  The library's debug switch
 makes the TMA producer skip its first K-tile load (a load that never
 arrives), so the consumers' waits run out: the kernel must then set the
-device error word, leave every loop, free its tensor memory and return, and
-refcache_status() must report REFCACHE_ERR_TIMEOUT -- no trap, no hang, and
-the context stays usable for the next, correct call.
+device error word (and the launching cache's own word), leave every loop,
+free its tensor memory and return, and refcache_status() (and the cache's
+refcache_cache_status()) must report REFCACHE_ERR_TIMEOUT -- no trap, no
+hang, and the context stays usable for the next, correct call.
 """
 import pytest
 import torch
@@ -54,19 +55,25 @@ def test_pair_kernel_wait_timeout_is_reported_and_context_survives(cache_dtype):
     seg = rcb.Segments.from_workload(w)
     H, D = w.num_heads, w.head_dim
     cache = rcb.RefCache(seg, device="cuda:0", cache_dtype=cache_dtype)
+    other = rcb.RefCache(seg, device="cuda:0", cache_dtype=cache_dtype)  # a second cache on the device
     qs, ks, vs = (t.cuda() for t in workloads.static_qkv(w))
     ql, kl, vl = (t.cuda() for t in workloads.live_qkv(w))
     o_s = torch.empty_like(qs)
     cache.build(0, qs, ks, vs, o_s)
+    other.build(0, qs, ks, vs, o_s)
     o_ref = torch.empty_like(ql)
     cache.step(0, ql, kl, vl, o_ref)
     torch.cuda.synchronize()
-    assert rcb.status() == rcb.OK
+    assert rcb.status() == rcb.OK and cache.status() == rcb.OK and other.status() == rcb.OK
     o = torch.zeros_like(ql)
     old = rcb.set_wait_timeout_ns(50_000_000)  # 50 ms
     try:
         rcb.debug_skip_first_load(True)
         cache.step(0, ql, kl, vl, o)
+        # the fault is this cache's: its own word says so, the other cache's does not
+        assert cache.status() == rcb.ERR_TIMEOUT
+        assert "this cache" in rcb.last_error()
+        assert cache.status() == rcb.OK and other.status() == rcb.OK
         assert rcb.status() == rcb.ERR_TIMEOUT
         assert "wait ran out" in rcb.last_error()
         assert rcb.status() == rcb.OK
