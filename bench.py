@@ -306,6 +306,7 @@ def run_ours(args, ws, rank, local):
         sustained figure was measured at a lower, power-capped clock)."""
         a = flops / secs / 1e12
         return {"achieved": a, "peak": peak, "unit": "TFLOP/s", "frac": a / peak}
+    traffic = recorded_traffic(w.name, args.kernel) if args.cache == "bf16" else None
     for entry in (sweep or []) + ([ragged] if ragged else []):
         for key in ("step", "prefill", "full"):
             if f"{key}_tflops" in entry:
@@ -361,7 +362,11 @@ def run_ours(args, ws, rank, local):
                               "1.4 GHz; this kernel's timed region runs near 2 GHz, so it is context only",
             "nominal_at_clock": nominal_at_clock(achieved, clocks.get("sm_mhz"), sms, peak_mult),
             "exp_floor": exp_floor(acc.step_units(w.requests) * H, t_step, clocks.get("sm_mhz"), sms),
-            "traffic": recorded_traffic(w.name, args.kernel) if args.cache == "bf16" else None,
+            "traffic": traffic,
+            # DRAM bytes of one launch (ncu record) over this run's step time: the
+            # cache and live streams' achieved bandwidth against the measured copy rate
+            "dram_gbs": traffic / t_step / 1e9 if traffic else None,
+            "dram_frac_of_hbm": traffic / t_step / 1e9 / pk["hbm_gbs"] if traffic else None,
             "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum, one step_attention launch"
                               " (profiles/); null when the kernel sources changed since",
             "algorithmic_bytes": 2 * (seg.live_rows * H * D * 2) * 2
