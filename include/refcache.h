@@ -292,10 +292,6 @@ REFCACHE_API int full_attention(int batch, int num_heads, int head_dim, const in
  *     REFCACHE_ERR_INVALID_ARG and a message naming the limit.
  *   - The first call on each device looks up the array's device address with
  *     that device current (a one-time set-up).
- *   - Not capturable in a CUDA graph: each call copies its work list from a
- *     host staging array (pageable memory) to the device array, which a stream
- *     capture does not accept, and a replay would reread whatever the last
- *     call left there.
  *   - Every call rewrites the whole work list it uses, so no state carries
  *     over, but all calls share the one array: calls whose kernels overlap on
  *     the GPU (different streams, or other threads) race.  Order them on one
