@@ -117,6 +117,9 @@ struct Cfg {
   static constexpr int kProducerWarp = kSoftmaxWarps, kMmaWarp = kSoftmaxWarps + 1, kGateWarp = kSoftmaxWarps + 2;
   static constexpr int kThreads = 32 * (kSoftmaxWarps + 3);
   static constexpr int kWarpArrivals = 2 * kSoftmaxWarps;  // p_full / q8_full: every softmax warp of both CTAs
+  // warps that take each item from the ring (work counter): the leader's
+  // gate and softmax warps, the follower's producer and softmax warps
+  static constexpr int kItemTakers = 2 + 2 * kSoftmaxWarps;
   static constexpr int kStages = kBN == 128 ? 4 : 3;     // ring stages (shared memory: 2 Q + stages <= 227 KB)
   static constexpr uint32_t kKBox = (kBN / 2) * 128;     // one K box: kBN / 2 rows x 128 bytes
   static constexpr uint32_t kKHalf = 2 * kKBox;          // this CTA's kBN / 2 keys x 128 d of a K tile
@@ -135,6 +138,7 @@ constexpr uint32_t kKHalf8 = 64 * 128;   // 8 KB: this CTA's 64 keys x 128 d of 
 constexpr uint32_t kVHalf8 = 64 * 128;   // 8 KB: this CTA's 64 d x 128 keys of an E4M3 V^T tile
 constexpr uint32_t kQ8Tile = 128 * 128;  // this CTA's 128 query rows as E4M3
 constexpr int kScaleSlots = 8;           // ring of per-tile scales of cached tiles (E4M3 kernel)
+constexpr int kItemSlots = 4;            // ring of items taken from the work counter
 
 template <bool kF8, int kBN>
 struct SmemT {
@@ -149,7 +153,8 @@ struct SmemT {
   static constexpr int kQFull = 0, kQEmpty = 2, kStageFull = 4, kPairDone = 4 + kStages,
                        kPFull = kPairDone + kPairDoneBars, kMmaDone = kPFull + 2, kQ8Full = kMmaDone + 1,
                        kLXFull = kQ8Full + 1, kScaleFull = kLXFull + 1, kScaleEmpty = kScaleFull + kScaleSlots,
-                       kNumBars = kScaleEmpty + kScaleSlots;
+                       kItemFull = kScaleEmpty + kScaleSlots, kItemEmpty = kItemFull + kItemSlots,
+                       kNumBars = kItemEmpty + kItemSlots;
   static constexpr uint32_t kTmemHolder = kBars + 8 * kNumBars;
   static constexpr uint32_t kAbort = kTmemHolder + 4;
   // load record of each CTA of the pair (leader's copy read at teardown):
@@ -157,7 +162,11 @@ struct SmemT {
   // (kStages) | loads per Q buffer (2)]
   static constexpr uint32_t kRecWords = 2 * kStages + 2;
   static constexpr uint32_t kLoadRec = kAbort + 4;
-  static constexpr uint32_t kUsed = kLoadRec + 2 * kRecWords * 4;
+  // ring of taken items (work counter): slot k % kItemSlots holds item k of
+  // this cluster (-1: none left); the gate warp passes the MMA warp its item
+  static constexpr uint32_t kItemRing = kLoadRec + 2 * kRecWords * 4;
+  static constexpr uint32_t kGateItem = kItemRing + 4 * kItemSlots;
+  static constexpr uint32_t kUsed = kGateItem + 4;
   static constexpr uint32_t kMaxDynamic = 232448;
   static constexpr uint32_t kDynamic = kUsed + 1024 < kMaxDynamic ? kUsed + 1024 : kMaxDynamic;
   static_assert(kUsed <= kMaxDynamic, "shared-memory layout too large");
@@ -213,6 +222,17 @@ __device__ __forceinline__ bool wait_cl_warp(uint32_t bar, uint32_t parity, cons
   const bool ok = wait_cl(bar, parity, c, where);
   return __all_sync(0xffffffffu, ok);
 }
+// Work counter [next item, clusters done]: this cluster has finished (every
+// item it took is done or abandoned); the last cluster resets both words for
+// the next launch, which reads them only after this grid has completed.
+__device__ __forceinline__ void work_done(int* work, int n_clusters) {
+  __threadfence();
+  if (atomicAdd(work + 1, 1) == n_clusters - 1) {
+    __threadfence();
+    atomicExch(work, 0);
+    atomicExch(work + 1, 0);
+  }
+}
 }  // namespace tc2
 
 template <bool kF8, int kBN>
@@ -260,6 +280,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
   // Both CTAs of a pair get the same layout, so both leave here together.
   if (base - raw + L::kUsed > L::kDynamic) {
     if (threadIdx.x == 0) tc::report_timeout(args.status, 99);
+    if (threadIdx.x == 0 && leader && args.work != nullptr) tc2::work_done(args.work, n_clusters);
     return;
   }
 
@@ -277,6 +298,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
     for (int s = 0; s < tc2::kScaleSlots; ++s) {
       mbar_init(bar(L::kScaleFull + s), 1);
       mbar_init(bar(L::kScaleEmpty + s), Cfg::kSoftmaxWarps);
+    }
+    for (int s = 0; s < tc2::kItemSlots; ++s) {
+      mbar_init(bar(L::kItemFull + s), 1);
+      mbar_init(bar(L::kItemEmpty + s), Cfg::kItemTakers);
     }
     *abort_flag = 0;
     fence_barrier_init();
@@ -298,6 +323,43 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
   const uint32_t tmem = *tmem_holder;
   const Ctl ctl{abort_flag, args.timeout_ns, args.status};
   auto lbar = [&](int i) -> uint32_t { return mapa_shared(bar(i), 0); };  // leader's barrier i
+  // Item k of this cluster (k = 0, 1, ...; -1 once there is none, -2 after a
+  // failed wait).  Static order: cluster + k * n_clusters.  With a work
+  // counter the leader's producer takes the next item of the list for each k
+  // (atomic increment) and writes it to ring slot k % kItemSlots of both CTAs;
+  // the other warps read it there.  A slot is reused once every taker has
+  // read it (item_empty, on the leader).
+  const bool dyn = args.work != nullptr;
+  volatile int* item_ring = reinterpret_cast<volatile int*>(base_ptr + L::kItemRing);
+  auto static_item = [&](int k) -> int {
+    const int64_t it = static_cast<int64_t>(cluster) + static_cast<int64_t>(k) * n_clusters;
+    return it < args.n_items ? static_cast<int>(it) : -1;
+  };
+  auto publish_item = [&](int k) -> int {  // leader's producer (one thread)
+    const int s = k % tc2::kItemSlots;
+    if (k >= tc2::kItemSlots &&
+        !wait_cl(bar(L::kItemEmpty + s), static_cast<uint32_t>(k / tc2::kItemSlots - 1) & 1u, ctl, 21))
+      return -2;
+    int it = atomicAdd(args.work, 1);
+    if (it >= args.n_items) it = -1;
+    item_ring[s] = it;
+    st_cluster_u32(mapa_shared(base + L::kItemRing + 4u * static_cast<uint32_t>(s), 1), static_cast<uint32_t>(it));
+    mbar_arrive(bar(L::kItemFull + s));
+    mbar_arrive_release_cluster(mapa_shared(bar(L::kItemFull + s), 1));
+    return it;
+  };
+  auto take_item = [&](int k, int where) -> int {  // one thread of a taking warp
+    const int s = k % tc2::kItemSlots;
+    if (!wait_cl(bar(L::kItemFull + s), static_cast<uint32_t>(k / tc2::kItemSlots) & 1u, ctl, where)) return -2;
+    const int it = item_ring[s];
+    mbar_arrive_release_cluster(lbar(L::kItemEmpty + s));
+    return it;
+  };
+  auto take_item_warp = [&](int k, int where) -> int {
+    int it = 0;
+    if (lane == 0) it = dyn ? take_item(k, where) : static_item(k);
+    return __shfl_sync(0xffffffffu, it, 0);
+  };
 
   if (warp == Cfg::kProducerWarp) {
     // ------------------------------------------------------------ producer (both CTAs)
@@ -370,7 +432,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
         ++g;
         return true;
       };
-      for (int item = cluster; item < args.n_items; item += n_clusters) {
+      for (int k = 0;; ++k) {
+        const int item = !dyn ? static_item(k) : leader ? publish_item(k) : take_item(k, 18);
+        if (item == -2) goto producer_done;
+        if (item < 0) break;
         decode_item(args, item, tk, head);
         const int nkv = tc2::n_key_tiles<kBN>(tk, na);
         if (nkv == 0) continue;
@@ -427,12 +492,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
       };
       bool issued = false;
       int g = 0, t0 = 0, qi = 0;
-      for (int item = cluster; item < args.n_items; item += n_clusters) {
+      const volatile int* gate_item = reinterpret_cast<const volatile int*>(base_ptr + L::kGateItem);
+      for (;;) {
+        // the gate warp names the next item with key tiles at this handshake;
+        // none left (or a failed wait) ends both warps
+        if (bar_red_or(tc2::kGateBarrier, 64, false)) goto mma_done;
         Task tk;
         int head, na;
-        decode_item(args, item, tk, head);
+        decode_item(args, *gate_item, tk, head);
         const int nkv = tc2::n_key_tiles<kBN>(tk, na);
-        if (nkv == 0) continue;
         const int qb = qi & 1;
         const uint64_t qd = qdesc0 + ((static_cast<uint32_t>(qb) * kQTile) >> 4);
         // groups G, G + 1: S_0, S_1 (the gate warp has seen the Q tile and stage g land)
@@ -536,12 +604,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
     // failed wait is passed on through the handshake, after which both leave.
     if (leader) {
       int g = 0, t0 = 0, qi = 0, q8i = 0;
-      for (int item = cluster; item < args.n_items; item += n_clusters) {
+      volatile int* gate_item = reinterpret_cast<volatile int*>(base_ptr + L::kGateItem);
+      for (int k = 0;; ++k) {
+        const int item = take_item_warp(k, 19);
         Task tk;
-        int head, na;
-        decode_item(args, item, tk, head);
-        const int nkv = tc2::n_key_tiles<kBN>(tk, na);
-        if (nkv == 0) continue;
+        int head = 0, na = 0, nkv = 0;
+        if (item >= 0) {
+          decode_item(args, item, tk, head);
+          nkv = tc2::n_key_tiles<kBN>(tk, na);
+          if (nkv == 0) continue;
+        }
+        // the MMA warp takes the item from here; the end of the list, or a
+        // failed wait, ends both warps
+        if (lane == 0) *gate_item = item;
+        if (bar_red_or(tc2::kGateBarrier, 64, item < 0)) goto gate_done;
         // the first cached tile's S also needs the E4M3 Q tile of both CTAs
         const bool q8 = kF8 && nkv > na;
         const uint32_t q8_parity = static_cast<uint32_t>(q8i) & 1u;
@@ -591,7 +667,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
     auto wait_group = [&](int g, int where) -> bool {
       return wait_cl_warp(bar(L::kPairDone + (g & 3)), group_parity(g), ctl, where);
     };
-    for (int item = cluster; item < args.n_items; item += n_clusters) {
+    for (int k = 0;; ++k) {
+      const int item = take_item_warp(k, 20);
+      if (item == -2) goto softmax_done;
+      if (item < 0) break;
       Task tk;
       int head;
       decode_item(args, item, tk, head);
@@ -960,6 +1039,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
   }
   // the follower leaves only once the leader has seen every load of the pair land
   cluster_sync();
+  if (dyn && leader && threadIdx.x == 0) tc2::work_done(args.work, n_clusters);
 }
 
 }  // namespace rc

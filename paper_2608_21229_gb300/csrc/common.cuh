@@ -57,6 +57,11 @@ struct AttnArgs {
   const __nv_bfloat16* kb;
   const __nv_bfloat16* vb;
   int* status;  // the launching cache's own error word (null: the device word only)
+  // CTA-pair kernel: null = static order (cluster c takes items c, c + n, ...);
+  // else [next item, clusters done], zero at launch: items are taken in list
+  // order by whichever cluster is free, and the last cluster to finish resets
+  // both words
+  int* work;
 };
 
 // One item whose key range was split into parts: the combine kernel merges

@@ -16,7 +16,6 @@
 #include <cstring>
 #include <functional>
 #include <mutex>
-#include <queue>
 #include <string>
 #include <vector>
 
@@ -55,6 +54,7 @@ int cuda_fail(cudaError_t e, const char* what) {
 }
 
 constexpr int kMaxDevices = 64;
+constexpr int kWorkOffset = 32;  // ints from a cache's error word to its work counter (a line of its own)
 
 struct DeviceInfo {
   bool checked = false;
@@ -298,6 +298,7 @@ struct Operands {
   void* o;
   float* lse;
   int* status = nullptr;  // the cache's own error word, if the launch is for a cache
+  int* work = nullptr;    // work counter of the CTA-pair kernel (two ints, zero between launches), or null
 };
 
 // Key range B as an E4M3 cache (cache_fp8.cuh): codes of K [rows_pad, H, 128],
@@ -372,6 +373,7 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
   a.rows_per_task = task_rows(D);
   a.timeout_ns = g_timeout_ns.load();
   a.status = op.status;
+  a.work = op.work;
   a.q = static_cast<const __nv_bfloat16*>(op.q);
   a.ka = static_cast<const __nv_bfloat16*>(op.ka);
   a.va = static_cast<const __nv_bfloat16*>(op.va);
@@ -502,40 +504,18 @@ void plan_items(const std::vector<Task>& tasks, int H, int clusters, int tile, s
   items->insert(items->end(), parts.begin(), parts.end());
 }
 
-// Lays a per-item list (longest items first) out for a persistent grid of
-// `clusters` CTA pairs, pair c taking slots c, c + clusters, c + 2 clusters,
-// ...: each item goes to the pair with the least work so far (longest
-// processing time first, ties to the lower pair), in the list's order, and
-// slots a pair does not need are empty tasks (no rows, no keys).  Work = MMA
-// groups: key tiles + 2.  Only the order changes, not any item's arithmetic.
-std::vector<Task> lpt_layout(const std::vector<Task>& items, int clusters, int tile) {
-  const int n = static_cast<int>(items.size());
-  const int c = std::min(n, clusters);
-  if (c <= 1) return items;
-  std::vector<int> order(n);
-  for (int i = 0; i < n; ++i) order[i] = i;
+// Orders a per-item list for the CTA-pair kernel, which hands items out in
+// list order to whichever CTA pair is free (a work counter): longest items
+// first (MMA groups: key tiles + 2), items of equal length in their order
+// (head-major, so that the pairs running at the same time share few heads'
+// K/V tiles in L2).  Only the order changes, not any item's arithmetic.
+std::vector<Task> longest_first(std::vector<Task> items, int tile) {
   auto groups = [&](const Task& t) -> int64_t {
     const int64_t nkv = (t.a_len + tile - 1) / tile + (t.b_len + tile - 1) / tile;
     return nkv > 0 ? nkv + 2 : 0;
   };
-  std::stable_sort(order.begin(), order.end(),
-                   [&](int x, int y) { return groups(items[x]) > groups(items[y]); });
-  using Load = std::pair<int64_t, int>;
-  std::priority_queue<Load, std::vector<Load>, std::greater<Load>> pq;
-  for (int i = 0; i < c; ++i) pq.push({0, i});
-  std::vector<std::vector<int>> per(c);
-  for (int i : order) {
-    const Load l = pq.top();
-    pq.pop();
-    per[l.second].push_back(i);
-    pq.push({l.first + groups(items[i]), l.second});
-  }
-  size_t depth = 0;
-  for (const auto& v : per) depth = std::max(depth, v.size());
-  std::vector<Task> out(static_cast<size_t>(c) * depth, Task{});
-  for (int p = 0; p < c; ++p)
-    for (size_t k = 0; k < per[p].size(); ++k) out[p + k * c] = items[per[p][k]];
-  return out;
+  std::stable_sort(items.begin(), items.end(), [&](const Task& x, const Task& y) { return groups(x) > groups(y); });
+  return items;
 }
 
 // Work list of full_attention_noalloc: a fixed array in static device memory
@@ -547,7 +527,8 @@ Task g_noalloc_host[REFCACHE_NOALLOC_MAX_TASKS];  // host staging, guarded by g_
 
 struct FullScratch {
   Task* buf = nullptr;
-  size_t cap = 0;  // tasks
+  size_t cap = 0;      // tasks
+  int* work = nullptr;  // work counter, after the tasks
 };
 FullScratch g_full[kMaxDevices];
 std::mutex g_full_mu;
@@ -571,6 +552,7 @@ struct refcache {
   int n_build_slot = 0;
   int64_t anchor_rows = 0;
   int* d_status = nullptr;  // this cache's error word (device int), see refcache_cache_status
+  int* d_work = nullptr;    // work counter of its CTA-pair launches (in the same 256-byte region)
   Task* d_step = nullptr;
   int n_step = 0;
   CopySeg* d_copy = nullptr;
@@ -692,7 +674,7 @@ int cache_plan(int num_layers, int mode_flags, const refcache_segments_t* seg, r
   off = align_up(off + cp.size() * sizeof(CopySeg), 256);
   off = align_up(off + qt.size() * sizeof(QuantTile), 256);
   off = align_up(off + bs.size() * sizeof(Task), 256);
-  off = align_up(off + sizeof(int), 256);  // the cache's error word
+  off = align_up(off + sizeof(int), 256);  // the cache's error word and work counter
   const size_t layer_bytes = f8 ? fp8_layer_bytes(off8[B], H, D) : 2 * slot_elems * sizeof(__nv_bfloat16);
   const size_t total = off + static_cast<size_t>(num_layers) * layer_bytes;
   if (h) {
@@ -750,31 +732,29 @@ int check_ptrs(std::initializer_list<const void*> ps, int64_t rows, const char* 
 // items are never split: each runs whole on one CTA pair, so a request's
 // prefill outputs depend on its own (N_ST, N_R) only -- not on the other
 // requests of the batch, nor on the device's SM count -- and the cached block
-// is reproduced bit for bit (Sec. 3.3).  Both are laid out by lpt_layout.
+// is reproduced bit for bit (Sec. 3.3).  Both are ordered by longest_first.
 int plan_split_items(refcache* h, DeviceInfo* info, const std::vector<Task>& bt, const std::vector<Task>& st) {
   // planned for the step kernel selected now (key tiles of tc2_tile(); the
-  // parts and the layout stay correct, only less even, if another tile size
+  // split and the order stay correct, only less even, if another tile size
   // or grid runs them)
   const bool f8 = h->f8 && h->rows_pad > 0;
   const int tile = tc2_tile(f8), tile_b = tc2_tile(false);
-  int clusters = 0, clusters_b = 0;
+  int clusters = 0;
   int rc = f8 ? tc2_clusters<true, 128>(info, &clusters)
               : tile == 128 ? tc2_clusters<false, 128>(info, &clusters) : tc2_clusters<false, 192>(info, &clusters);
-  if (rc) return rc;
-  rc = tile_b == 128 ? tc2_clusters<false, 128>(info, &clusters_b) : tc2_clusters<false, 192>(info, &clusters_b);
   if (rc) return rc;
   std::vector<Task> si, bi;
   std::vector<CombineJob> sj;
   int parts = 0;
   plan_items(st, h->H, clusters, tile, &si, &sj, &parts);
-  si = lpt_layout(si, clusters, tile);
+  si = longest_first(std::move(si), tile);
   for (int hd = 0; hd < h->H; ++hd)
     for (Task t : bt) {
       t.head = hd;
       t.part = 0;
       bi.push_back(t);
     }
-  bi = lpt_layout(bi, clusters_b, tile_b);
+  bi = longest_first(std::move(bi), tile_b);
   const int rows = task_rows(h->D);
   size_t off = 0;
   const size_t o_bi = off;
@@ -879,6 +859,7 @@ int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refca
   h->d_build_slot = reinterpret_cast<Task*>(h->mem + off);
   off = align_up(off + bs.size() * sizeof(Task), 256);
   h->d_status = reinterpret_cast<int*>(h->mem + off);
+  h->d_work = h->d_status + kWorkOffset;
   off = align_up(off + sizeof(int), 256);
   h->slots = reinterpret_cast<__nv_bfloat16*>(h->mem + off);
   h->slots8 = h->mem + off;
@@ -890,7 +871,8 @@ int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refca
     e = cudaMemcpy(h->d_qtiles, qt.data(), qt.size() * sizeof(QuantTile), cudaMemcpyHostToDevice);
   if (!bs.empty() && e == cudaSuccess)
     e = cudaMemcpy(h->d_build_slot, bs.data(), bs.size() * sizeof(Task), cudaMemcpyHostToDevice);
-  if (e == cudaSuccess) e = cudaMemset(h->d_status, 0, sizeof(int));
+  if (e == cudaSuccess) e = cudaMemset(h->d_status, 0, 256);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();  // zero before any stream's first launch
   if (e != cudaSuccess) {
     if (h->owns) cudaFree(h->mem);
     delete h;
@@ -995,7 +977,7 @@ int refcache_build(refcache_t* h, int layer, const void* q_static, const void* k
     cj.rows = h->cache_rows;
   }
   Operands op{q_static, h->static_rows, k_static, v_static, h->static_rows, nullptr, nullptr, 0, o_static, lse_static,
-              h->d_status};
+              h->d_status, h->d_work};
   rc = run_attention(h->d_build, h->n_build, h->H, h->D, op, softmax_scale, info, s,
                      h->build_items.items ? &h->build_items : nullptr, nullptr, h->n_copy > 0 ? &cj : nullptr);
   if (rc) return rc;
@@ -1031,7 +1013,7 @@ int refcache_build_in_slot(refcache_t* h, int layer, const void* q_static, const
               range_b ? h->cache_rows : 0,
               o_static,
               lse_static,
-              h->d_status};
+              h->d_status, h->d_work};
   rc = run_attention(h->d_build_slot, h->n_build_slot, h->H, h->D, op, softmax_scale, info,
                      static_cast<cudaStream_t>(stream));
   if (rc) return rc;
@@ -1060,7 +1042,7 @@ int step_attention(refcache_t* h, int layer, const void* q_live, const void* k_l
     refcache_kv_ptr(h, layer, &kslot, &vslot, nullptr);
   }
   Operands op{q_live, h->live_rows, k_live, v_live, h->live_rows, kslot, vslot, h->cache_rows, o_live, lse_live,
-              h->d_status};
+              h->d_status, h->d_work};
   return run_attention(h->d_step, h->n_step, h->H, h->D, op, softmax_scale, info, static_cast<cudaStream_t>(stream),
                        h->step_items.items ? &h->step_items : nullptr, use_f8 ? &f8 : nullptr);
 }
@@ -1086,6 +1068,7 @@ int full_attention(int batch, int num_heads, int head_dim, const int32_t* cu_seq
   if (tasks.empty()) return REFCACHE_OK;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   Task* d_tasks = nullptr;
+  int* work = nullptr;
   {
     std::lock_guard<std::mutex> lk(g_full_mu);
     FullScratch& fs = g_full[dev];
@@ -1098,15 +1081,19 @@ int full_attention(int batch, int num_heads, int head_dim, const int32_t* cu_seq
         fs.cap = 0;
       }
       const size_t cap = std::max<size_t>(tasks.size(), 1024);
-      cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&fs.buf), cap * sizeof(Task));
+      cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&fs.buf), cap * sizeof(Task) + 256);
       if (e != cudaSuccess) return fail(REFCACHE_ERR_OOM, "cudaMalloc(work list): %s", cudaGetErrorString(e));
       fs.cap = cap;
+      fs.work = reinterpret_cast<int*>(fs.buf + cap);
+      e = cudaMemsetAsync(fs.work, 0, 256, s);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync(work counter)");
     }
     d_tasks = fs.buf;
+    work = fs.work;
     cudaError_t e = cudaMemcpyAsync(d_tasks, tasks.data(), tasks.size() * sizeof(Task), cudaMemcpyHostToDevice, s);
     if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync(work list)");
   }
-  Operands op{q, rows, k, v, rows, nullptr, nullptr, 0, o, lse};
+  Operands op{q, rows, k, v, rows, nullptr, nullptr, 0, o, lse, nullptr, work};
   return run_attention(d_tasks, static_cast<int>(tasks.size()), num_heads, head_dim, op, softmax_scale, info, s);
 }
 
