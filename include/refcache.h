@@ -161,8 +161,13 @@ REFCACHE_API size_t refcache_bytes(int num_layers, int mask_mode, const refcache
  * the caller, not freed).  Synchronous.  *out is set only on success.
  *
  * For head_dim 128 it also plans, for the current device, the per-item work
- * lists of the prefill and the step, each (query tile, head) item assigned to
- * the CTA pair with the least work so far (longest first).  When the step's
+ * lists of the prefill and the step, (query tile, head) items longest first;
+ * a launch hands them out in that order to whichever CTA pair is free,
+ * through a work counter kept in the cache's memory (reset by the launch
+ * itself when it ends), so the pair that computes an item varies but its
+ * arithmetic does not.  full_attention does the same with a counter kept
+ * beside its work list; full_attention_noalloc takes items in a fixed order
+ * (the same results, bit for bit).  When the step's
  * items do not fill the last round of the GPU's CTA pairs evenly, the items of
  * that round are split by key range into 2-8 parts whose outputs a combine
  * kernel merges.  These lists and an fp32 workspace for the parts (parts x 256

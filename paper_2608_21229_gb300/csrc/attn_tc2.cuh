@@ -34,8 +34,11 @@
 // One softmax warp per SM sub-partition leaves the MMA warp's sub-partition
 // with a single busy warp beside it, and a row needs no partner thread.
 // An item is a task of up to 256 query rows: CTA r takes rows
-// [128 r, 128 r + 128).  Items are taken cluster by cluster from a per-item
-// list laid out on the host, or head-major from the task list.
+// [128 r, 128 r + 128).  Items come from a per-item list ordered on the host
+// or, head-major, from the task list: with a work counter each CTA pair takes
+// the next item of the list whenever it starts one (the leader's producer
+// takes it and passes it on through a ring in shared memory), else pair c
+// takes items c, c + n_pairs, ...
 //
 // Work is done item by item (an item = a task of up to 256 rows x one
 // head).  An item with n key tiles is a sequence of n + 2 MMA groups:

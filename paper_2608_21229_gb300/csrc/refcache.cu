@@ -167,7 +167,7 @@ int64_t task_cost(const Task& t) {
   return static_cast<int64_t>((t.q_rows + 127) / 128) * ((t.a_len + 127) / 128 + (t.b_len + 127) / 128);
 }
 
-// Longest tasks first: the persistent CTAs take items round-robin.
+// Longest tasks first: the order in which the persistent CTAs take items.
 void order_tasks(std::vector<Task>& v) {
   std::stable_sort(v.begin(), v.end(), [](const Task& x, const Task& y) { return task_cost(x) > task_cost(y); });
 }
