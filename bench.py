@@ -247,6 +247,9 @@ def run_ours(args, ws, rank, local):
     st = rcb.status()
     if st != rcb.OK:
         raise RuntimeError(f"device error during warm-up: {rcb.last_error()}")
+    # the exponential unit's rate on this GPU (the softmax's secondary limit),
+    # measured before the timed region
+    ex2_rate = rcb.ex2_rate()
 
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -361,7 +364,7 @@ def run_ours(args, ws, rank, local):
             "sustained_note": "the sustained peak was measured at a power-capped median SM clock of about "
                               "1.4 GHz; this kernel's timed region runs near 2 GHz, so it is context only",
             "nominal_at_clock": nominal_at_clock(achieved, clocks.get("sm_mhz"), sms, peak_mult),
-            "exp_floor": exp_floor(acc.step_units(w.requests) * H, t_step, clocks.get("sm_mhz"), sms),
+            "exp_floor": exp_floor(acc.step_units(w.requests) * H, t_step, clocks.get("sm_mhz"), sms, ex2_rate),
             "traffic": traffic,
             # DRAM bytes of one launch (ncu record) over this run's step time: the
             # cache and live streams' achieved bandwidth against the measured copy rate
@@ -397,20 +400,19 @@ def nominal_at_clock(achieved, sm_mhz, sms, mult=1.0):
             "frac": achieved / ceiling}
 
 
-# Exponentials per clock per SM of ex2.approx.f32 (MUFU), measured on this
-# GPU by a probe kernel: one warp instruction per 4 cycles per sub-partition.
-MUFU_EX2_PER_CLK_PER_SM = 32
-
-
-def exp_floor(units, secs, sm_mhz, sms):
+def exp_floor(units, secs, sm_mhz, sms, ex2_per_clk_per_sm):
     """The secondary ALU limit: one exponential per visible (query, key) pair
-    of one head against the MUFU rate at the sampled clock."""
+    of one head against the exponential unit's rate (ex2.approx.f32 per clock
+    per SM, measured on this GPU by the library's probe kernel) at the sampled
+    clock."""
     if not sm_mhz:
         return None
-    floor = units / (MUFU_EX2_PER_CLK_PER_SM * sms * sm_mhz * 1e6)
-    return {"exps": units, "ex2_per_clk_per_sm": MUFU_EX2_PER_CLK_PER_SM, "sm_mhz": sm_mhz,
-            "floor_ms": floor * 1e3, "frac_of_step": floor / secs,
-            "note": "MUFU time the exponentials need at the sampled clock, as a share of the step"}
+    floor = units / (ex2_per_clk_per_sm * sms * sm_mhz * 1e6)
+    return {"exps": units, "ex2_per_clk_per_sm": ex2_per_clk_per_sm,
+            "ex2_rate_source": "measured on this GPU (refcache_ex2_rate: one CTA per SM, 8 warps x 8 independent "
+                               "ex2.approx.f32 chains, clock64)",
+            "sm_mhz": sm_mhz, "floor_ms": floor * 1e3, "frac_of_step": floor / secs,
+            "note": "time the exponentials need at the sampled clock, as a share of the step"}
 
 
 def gpu_randn_bf16(shape, seed: int, dev):

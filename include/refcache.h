@@ -344,6 +344,18 @@ REFCACHE_API int refcache_set_kernel(int kernel);
  */
 REFCACHE_API void refcache_debug_skip_first_load(int on);
 
+/*
+ * Diagnostic: the rate of the GPU's exponential unit (ex2.approx.f32, the
+ * special-function unit) on the current device, in exponentials per clock per
+ * SM (median over the SMs), written to *per_clk_per_sm (host).  The softmax
+ * of the attention kernels evaluates one exponential per visible (query, key)
+ * pair of one head; this rate gives that work's floor beside the tensor-core
+ * roofline.  The paper has no counterpart.  Runs one short kernel (one CTA
+ * per SM, about 0.1 ms) on `stream` and synchronises it; allocates nothing.
+ * Returns REFCACHE_ERR_INVALID_ARG for a NULL pointer.
+ */
+REFCACHE_API int refcache_ex2_rate(double* per_clk_per_sm, void* stream);
+
 /* Copy the calling thread's last error message into buf (NUL-terminated); returns its length. */
 REFCACHE_API int refcache_last_error(char* buf, size_t n);
 

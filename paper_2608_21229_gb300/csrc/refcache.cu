@@ -25,6 +25,7 @@
 #include "attn_tc2.cuh"
 #include "attn_combine.cuh"
 #include "cache_fp8.cuh"
+#include "mufu_rate.cuh"
 
 using rc::AttnArgs;
 using rc::CombineJob;
@@ -1198,6 +1199,30 @@ int refcache_set_kernel(int kernel) {
 }
 
 void refcache_debug_skip_first_load(int on) { g_dbg_skip.store(on ? 1 : 0); }
+
+int refcache_ex2_rate(double* per_clk_per_sm, void* stream) {
+  if (!per_clk_per_sm) return fail(REFCACHE_ERR_INVALID_ARG, "per_clk_per_sm is NULL");
+  DeviceInfo* info = nullptr;
+  int rc = enter_device(nullptr, &info);
+  if (rc) return rc;
+  const int blocks = std::min(info->num_sms, rc::kEx2MaxBlocks);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaFuncSetAttribute(rc::ex2_rate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, rc::kEx2Smem);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(ex2_rate_kernel)");
+  rc::ex2_rate_kernel<<<blocks, rc::kEx2Threads, rc::kEx2Smem, s>>>(-1.0f);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "ex2_rate_kernel launch");
+  std::vector<long long> cyc(static_cast<size_t>(blocks));
+  e = cudaMemcpyFromSymbolAsync(cyc.data(), rc::g_ex2_cycles, cyc.size() * sizeof(long long), 0,
+                                cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_fail(e, "read ex2_rate_kernel cycles");
+  std::sort(cyc.begin(), cyc.end());
+  const long long med = cyc[cyc.size() / 2];
+  if (med <= 0) return fail(REFCACHE_ERR_CUDA, "ex2_rate_kernel measured no cycles");
+  *per_clk_per_sm = static_cast<double>(rc::kEx2Threads) * rc::kEx2Chains * rc::kEx2Iters / static_cast<double>(med);
+  return REFCACHE_OK;
+}
 
 int refcache_last_error(char* buf, size_t n) {
   if (buf && n > 0) {

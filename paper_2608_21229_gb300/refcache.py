@@ -31,7 +31,7 @@ EXPORTED = (
     "refcache_build", "step_attention", "full_attention", "refcache_status", "refcache_set_wait_timeout_ns",
     "refcache_set_kernel", "refcache_debug_skip_first_load", "refcache_last_error", "refcache_version",
     "full_attention_noalloc", "refcache_call_launches", "refcache_fp8_ptr", "refcache_build_in_slot",
-    "refcache_cache_status",
+    "refcache_cache_status", "refcache_ex2_rate",
 )
 NOALLOC_MAX_TASKS = 16384
 
@@ -91,6 +91,7 @@ def load(path: Optional[str] = None):
     L.refcache_set_wait_timeout_ns.restype = ctypes.c_uint64
     L.refcache_set_kernel.argtypes = [i32]
     L.refcache_debug_skip_first_load.argtypes = [i32]
+    L.refcache_ex2_rate.argtypes = [ctypes.POINTER(ctypes.c_double), vp]
     L.refcache_debug_skip_first_load.restype = None
     L.refcache_last_error.argtypes = [ctypes.c_char_p, ctypes.c_size_t]
     L.refcache_version.restype = ctypes.c_char_p
@@ -161,6 +162,14 @@ def debug_skip_first_load(on: bool = True) -> None:
 def status(stream=None) -> int:
     """Synchronise the stream and return the device error word as a status code."""
     return int(load().refcache_status(_stream(stream)))
+
+
+def ex2_rate(stream=None) -> float:
+    """Exponentials (ex2.approx.f32) per clock per SM measured on the current
+    device by the library's probe kernel."""
+    v = ctypes.c_double(0.0)
+    _check(load().refcache_ex2_rate(ctypes.byref(v), _stream(stream)))
+    return float(v.value)
 
 
 def version() -> str:

@@ -48,7 +48,7 @@ def test_workload_shapes():
 def test_bench_clock_ceilings():
     """The bench line's two clock-based figures: the tensor pipe's ceiling
     (8192 dense bf16 FLOPs per clock per SM) and the exponential floor (one
-    MUFU ex2 per visible pair, 32 per clock per SM), at a given clock."""
+    ex2 per visible pair at a given rate per clock per SM), at a given clock."""
     import bench
 
     n = bench.nominal_at_clock(1000.0, 2000.0, 152)
@@ -56,6 +56,8 @@ def test_bench_clock_ceilings():
     assert bench.nominal_at_clock(1000.0, None, 152) is None
     w = workloads.EDIT_1024_5REF
     exps = acc.step_units(w.requests) * w.num_heads
-    f = bench.exp_floor(exps, 1e-3, 2000.0, 152)
+    f = bench.exp_floor(exps, 1e-3, 2000.0, 152, 32.0)
     assert f["floor_ms"] == pytest.approx(exps / (32 * 152 * 2.0e9) * 1e3)
     assert f["frac_of_step"] == pytest.approx(f["floor_ms"] / 1.0)
+    assert bench.exp_floor(exps, 1e-3, 2000.0, 152, 16.0)["floor_ms"] == pytest.approx(2 * f["floor_ms"])
+    assert bench.exp_floor(exps, 1e-3, None, 152, 32.0) is None
