@@ -558,7 +558,7 @@ struct refcache {
   int n_step = 0;
   CopySeg* d_copy = nullptr;
   int n_copy = 0;
-  // per-item lists of the head-dim-128 kernel, laid out for the persistent
+  // per-item lists of the head-dim-128 kernel, ordered for the persistent
   // grid (the step's with split items), in a separate allocation:
   // [build items | step items | step jobs | part_o | part_lse]
   uint8_t* aux = nullptr;
