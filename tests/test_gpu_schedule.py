@@ -9,6 +9,8 @@ resets the counter for the next launch.  Checked through the C ABI:
   - launches with more items than CTA pairs and with fewer, interleaved on one
     stream and across two caches, repeat their bytes (an unreset counter
     would skip items and leave the NaN the outputs are filled with);
+  - two caches (each with its own counter) driven at the same time on two
+    streams give the bytes of the same calls made one after the other;
   - the same holds for the E4M3 cache's kernel.
 """
 import numpy as np
@@ -124,3 +126,26 @@ def test_e4m3_cache_step_repeats_its_bytes():
         assert np.array_equal(pu.bits(step().cpu()), first)
     torch.cuda.synchronize()
     assert rcb.status() == rcb.OK
+
+
+def test_two_caches_on_two_streams_at_once():
+    """Each cache has its own work counter, so launches of two caches may run
+    at the same time on two streams; their outputs equal those of the same
+    calls made one after the other."""
+    runs = {}
+    for name, w in (("a", workloads.EDIT_512_2REF), ("b", workloads.RAGGED_4REQ)):
+        cache, _, step = _cache_run(w)
+        runs[name] = (cache, step, pu.bits(step().cpu()))
+    torch.cuda.synchronize()
+    sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
+    outs = {"a": [], "b": []}
+    for _ in range(3):
+        for name, s in (("a", sa), ("b", sb)):
+            with torch.cuda.stream(s):
+                outs[name].append(runs[name][1]())
+    torch.cuda.synchronize()
+    assert rcb.status() == rcb.OK
+    for name in ("a", "b"):
+        assert runs[name][0].status() == rcb.OK
+        for o in outs[name]:
+            assert np.array_equal(pu.bits(o.cpu()), runs[name][2]), name
