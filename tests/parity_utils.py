@@ -142,3 +142,15 @@ def sampled_compare(run: GpuRun, seed=0, per_request=24, scale=None, heads=None)
         ref_o, ref_l = oracle_live_request(w, mode, b, run.static, run.live, scale, pairs)
         check_close(o_l[l0 + pairs[:, 0], pairs[:, 1]], ref_o, l_l[l0 + pairs[:, 0], pairs[:, 1]], ref_l,
                     f"step req {b} (sampled)")
+
+
+def guard_report(full: np.ndarray, guard: int, n: int, width: int, pattern: int):
+    """For a byte buffer laid out as [guard | n bytes of elements of `width`
+    bytes | guard], all set to `pattern` before a call: the guard bytes that
+    changed before and after the elements, and the elements that still hold
+    the pattern in every byte (never written)."""
+    before = int((full[:guard] != pattern).sum())
+    after = int((full[guard + n:] != pattern).sum())
+    words = full[guard:guard + n].reshape(-1, width)
+    untouched = int((words == pattern).all(axis=1).sum()) if n else 0
+    return before, after, untouched

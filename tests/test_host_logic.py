@@ -61,3 +61,22 @@ def test_bench_clock_ceilings():
     assert f["frac_of_step"] == pytest.approx(f["floor_ms"] / 1.0)
     assert bench.exp_floor(exps, 1e-3, 2000.0, 152, 16.0)["floor_ms"] == pytest.approx(2 * f["floor_ms"])
     assert bench.exp_floor(exps, 1e-3, None, 152, 32.0) is None
+
+
+def test_guard_report_finds_planted_writes():
+    """The canary check of tests/test_gpu_canary.py: bytes changed in either
+    guard and elements left unwritten are counted (planted on the CPU)."""
+    import numpy as np
+    import parity_utils as pu
+
+    g, n, pat = 64, 40, 0xA5
+    full = np.full(g + n + g, pat, dtype=np.uint8)
+    full[g:g + n] = 1                      # every element written
+    assert pu.guard_report(full, g, n, 4, pat) == (0, 0, 0)
+    full[g - 1] = 0                        # one byte before the buffer
+    full[g + n + 5] = 7                    # and one after
+    full[g + 8:g + 12] = pat               # one 4-byte element never written
+    assert pu.guard_report(full, g, n, 4, pat) == (1, 1, 1)
+    full[g + 12] = pat                     # a partly matching element is written
+    assert pu.guard_report(full, g, n, 4, pat)[2] == 1
+    assert pu.guard_report(full, g, n, 2, pat)[2] == 2
