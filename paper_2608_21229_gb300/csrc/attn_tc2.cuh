@@ -941,6 +941,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
         if (lane == 0) mbar_arrive_cluster(mapa_shared(bar(L::kPFull + b), 0));
       }
       {
+        // the row's place: the bf16 kernels read it again from the work list, so
+        // that it is not kept live through the tile loop
+        bool e_row_ok = row_ok;
+        int64_t e_grow = grow;
+        __nv_bfloat16* e_orow = orow;
+        int e_head = head, e_part = tk.part;
+        if constexpr (!kF8) {
+          Task et;
+          decode_item(args, item, et, e_head);
+          e_row_ok = prow < et.q_rows;
+          e_grow = static_cast<int64_t>(et.q_row0) + prow;
+          e_orow = args.out + e_grow * args.row_stride + static_cast<int64_t>(e_head) * D + ocol0;
+          e_part = et.part;
+        }
         if (!wait_group(G + nkv + 1, 10)) goto softmax_done;  // the item's last group
         tc_fence_after();
         float l_tot = l_run;
@@ -955,16 +969,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
         }
         const float inv_l = kF8 ? s_ref / l_tot : 1.0f / l_tot;
         const uint32_t t_o = tmem + lane_off + kColO + static_cast<uint32_t>(ocol0);
-        if (tk.part > 0) {
+        if (e_part > 0) {
           // a part of a split item: O / l in fp32 and m + log l to its workspace slot
-          const int64_t prow_ws = static_cast<int64_t>(tk.part - 1) * args.rows_per_task + prow;
+          const int64_t prow_ws = static_cast<int64_t>(e_part - 1) * args.rows_per_task + prow;
           float4* dst = reinterpret_cast<float4*>(args.part_o + prow_ws * D + ocol0);
 #pragma unroll
           for (int cc = 0; cc < kOC / 32; ++cc) {
             uint32_t o[32];
             tmem_ld32(t_o + 32u * cc, o);
             tmem_wait_ld(o);
-            if (row_ok) {
+            if (e_row_ok) {
 #pragma unroll
               for (int c = 0; c < 8; ++c)
                 dst[8 * cc + c] = make_float4(__uint_as_float(o[4 * c]) * inv_l, __uint_as_float(o[4 * c + 1]) * inv_l,
@@ -973,7 +987,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
             }
           }
           tc_fence_before();
-          if (row_ok && hh == 0) args.part_lse[prow_ws] = (m_run + log2f(l_tot)) * 0.69314718055994530942f;
+          if (e_row_ok && hh == 0) args.part_lse[prow_ws] = (m_run + log2f(l_tot)) * 0.69314718055994530942f;
           G += nkv + 2;
           continue;
         }
@@ -991,13 +1005,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
         // (the next arrival on p_full, after the next tile's P, tells the MMA
         // thread that these O reads are done)
         tc_fence_before();
-        if (row_ok) {
-          uint4* dst = reinterpret_cast<uint4*>(orow);
+        if (e_row_ok) {
+          uint4* dst = reinterpret_cast<uint4*>(e_orow);
 #pragma unroll
           for (int c = 0; c < kOC / 8; ++c)
             dst[c] = make_uint4(packed[4 * c], packed[4 * c + 1], packed[4 * c + 2], packed[4 * c + 3]);
           if (args.lse && hh == 0)
-            args.lse[grow * args.num_heads + head] = (m_run + log2f(l_tot)) * 0.69314718055994530942f;
+            args.lse[e_grow * args.num_heads + e_head] = (m_run + log2f(l_tot)) * 0.69314718055994530942f;
         }
       }
       G += nkv + 2;
