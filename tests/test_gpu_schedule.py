@@ -11,6 +11,8 @@ resets the counter for the next launch.  Checked through the C ABI:
     would skip items and leave the NaN the outputs are filled with);
   - two caches (each with its own counter) driven at the same time on two
     streams give the bytes of the same calls made one after the other;
+  - 240 launches of four kinds in rotation, with no host synchronisation
+    between them, all repeat the bytes of the first call of their kind;
   - the same holds for the E4M3 cache's kernel.
 """
 import numpy as np
@@ -149,3 +151,33 @@ def test_two_caches_on_two_streams_at_once():
         assert runs[name][0].status() == rcb.OK
         for o in outs[name]:
             assert np.array_equal(pu.bits(o.cpu()), runs[name][2]), name
+
+
+def test_counter_survives_many_launches():
+    """Many launches back to back with no host synchronisation between them:
+    steps of two caches and full attention of two sizes in a fixed rotation,
+    every output checked against the first call of its kind, bit for bit."""
+    a_cache, _, a_step = _cache_run(workloads.EDIT_512_2REF)
+    b_cache, _, b_step = _cache_run(workloads.RAGGED_4REQ)
+    big, small = _qkv(*BIG), _qkv(*SMALL)
+    calls = {
+        "a": a_step,
+        "b": b_step,
+        "big": lambda: _full(rcb.full_attention, *big)[0],
+        "small": lambda: _full(rcb.full_attention, *small)[0],
+    }
+    first = {k: pu.bits(f().cpu()) for k, f in calls.items()}
+    outs = []
+    for i in range(60):
+        for k in ("a", "big", "b", "small") if i % 2 == 0 else ("small", "b", "a", "big"):
+            outs.append((k, calls[k]()))
+        if len(outs) >= 40:  # compare in batches to bound the memory held
+            torch.cuda.synchronize()
+            for k, o in outs:
+                assert np.array_equal(pu.bits(o.cpu()), first[k]), k
+            outs = []
+    torch.cuda.synchronize()
+    for k, o in outs:
+        assert np.array_equal(pu.bits(o.cpu()), first[k]), k
+    assert rcb.status() == rcb.OK
+    assert a_cache.status() == rcb.OK and b_cache.status() == rcb.OK
