@@ -44,9 +44,10 @@
  *     cache, unless it is given memory, and for head_dim 128 a separate work
  *     list with a workspace for split items, see refcache_create) and
  *     full_attention (a per-device work-list buffer that it keeps and grows).
- *   - The refcache_build and step_attention calls of one cache share that
- *     workspace: issue them in stream order (one stream, or streams ordered
- *     by events), not concurrently.
+ *   - The refcache_build, refcache_build_in_slot and step_attention calls of
+ *     one cache share that workspace and the cache's work counter: issue them
+ *     in stream order (one stream, or streams ordered by events), not
+ *     concurrently.  Calls for different caches may run concurrently.
  *   - The head-dim-128 attention kernel and the merge of split items are
  *     launched as programmatic dependents of the previous kernel on the
  *     stream: they wait for it to complete before they read memory, and they
