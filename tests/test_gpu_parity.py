@@ -325,3 +325,27 @@ def test_rescale_path_full_compare(kernel, head_dim):
     w = workloads.Workload(f"growing_keys_d{head_dim}", 2, head_dim, (workloads.Request(16, 32, 200, 1500),), 13)
     run = pu.GpuRun(w, kernel=kernel, static=_growing_keys(w))
     pu.full_compare(run)
+
+
+@pytest.mark.parametrize("kernel,head_dim", [("tcgen05", 128), ("tcgen05_k128", 128), ("tcgen05", 64)])
+def test_many_requests_full_compare(kernel, head_dim):
+    """40 requests of uneven lengths (up to about 660 live and 600 cached rows) on 8 heads:
+    hundreds of work items of different sizes, several per CTA pair, handed
+    out by the work counter longest first; every output row compared with the
+    oracle."""
+    rng = np.random.default_rng(2024 + head_dim)
+    reqs = list(workloads.random_requests(rng, 40, max_len=600))
+    w = workloads.Workload(f"many_requests_{head_dim}", 8, head_dim, tuple(reqs), 17)
+    run = pu.GpuRun(w, mode="beyond", kernel=kernel)
+    pu.full_compare(run)
+
+
+def test_split_tail_items_full_compare():
+    """A step whose items all fall in the last round and are long enough to
+    split: one request of 768 live rows over 3000 cached rows on 8 heads is
+    24 items of 20 key tiles, each split into parts that run on separate CTA
+    pairs and are merged by the combine kernel; every output row against the
+    oracle, and the cache and prefill as well."""
+    w = workloads.Workload("split_tail_768x3000", 8, 128, (workloads.Request(64, 256, 512, 3000),), 19)
+    run = pu.GpuRun(w, mode="beyond", kernel="tcgen05")
+    pu.full_compare(run)
