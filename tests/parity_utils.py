@@ -29,8 +29,9 @@ class GpuRun:
     """One workload through the library: build of layer 0, one step, outputs on the CPU."""
 
     def __init__(self, w, mode="beyond", kernel="tcgen05", layer=0, step=0, num_layers=1, static=None, live=None,
-                 device="cuda:0"):
+                 device="cuda:0", scale=None):
         self.w, self.mode = w, mode
+        self.scale = scale  # softmax scale passed to the library (None: 1/sqrt(head_dim))
         rcb.set_kernel(kernel)
         self.seg = rcb.Segments.from_workload(w)
         self.static = static if static is not None else workloads.static_qkv(w, layer)
@@ -44,8 +45,8 @@ class GpuRun:
         self.lse_static = torch.full((self.seg.static_rows, H), float("nan"), dtype=torch.float32, device=dev)
         self.o_live = torch.full((self.seg.live_rows, H, D), float("nan"), dtype=torch.bfloat16, device=dev)
         self.lse_live = torch.full((self.seg.live_rows, H), float("nan"), dtype=torch.float32, device=dev)
-        self.cache.build(layer, qs, ks, vs, self.o_static, self.lse_static)
-        self.cache.step(layer, ql, kl, vl, self.o_live, self.lse_live)
+        self.cache.build(layer, qs, ks, vs, self.o_static, self.lse_static, scale=scale)
+        self.cache.step(layer, ql, kl, vl, self.o_live, self.lse_live, scale=scale)
         torch.cuda.synchronize()
         assert rcb.status() == rcb.OK, rcb.last_error()
         self.k_cache, self.v_cache = (t.cpu() for t in self.cache.kv(layer))
@@ -91,9 +92,10 @@ def check_close(gpu_o, ref_o, gpu_lse=None, ref_lse=None, what=""):
 
 
 def full_compare(run: GpuRun, scale=None):
-    """Every output row of both calls against the oracle."""
+    """Every output row of both calls against the oracle (at the run's softmax
+    scale unless one is given)."""
     w, mode = run.w, run.mode
-    scale = scale or 1.0 / math.sqrt(w.head_dim)
+    scale = scale or run.scale or 1.0 / math.sqrt(w.head_dim)
     o_s, l_s, o_l, l_l = f64(run.o_static), f64(run.lse_static), f64(run.o_live), f64(run.lse_live)
     coff = cache_offsets(w, mode)
     for b, r in enumerate(w.requests):

@@ -349,3 +349,18 @@ def test_split_tail_items_full_compare():
     w = workloads.Workload("split_tail_768x3000", 8, 128, (workloads.Request(64, 256, 512, 3000),), 19)
     run = pu.GpuRun(w, mode="beyond", kernel="tcgen05")
     pu.full_compare(run)
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("head_dim", [64, 128])
+@pytest.mark.parametrize("scale", [0.02, 0.3, 1.0])
+def test_softmax_scale_full_compare(kernel, head_dim, scale):
+    """Softmax scales other than 1/sqrt(d): nearly uniform weights (0.02) and
+    nearly one-hot rows whose running maximum moves often (1.0: scaled scores
+    with a standard deviation of sqrt(d)); prefill, cache and step against the
+    oracle at the same scale."""
+    rng = np.random.default_rng(int(scale * 1000) + head_dim)
+    reqs = list(workloads.random_requests(rng, 3, max_len=500))
+    w = workloads.Workload(f"scale_{scale}_{head_dim}", 3, head_dim, tuple(reqs), 23)
+    run = pu.GpuRun(w, mode="beyond", kernel=kernel, scale=scale)
+    pu.full_compare(run)
