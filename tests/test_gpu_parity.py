@@ -364,3 +364,43 @@ def test_softmax_scale_full_compare(kernel, head_dim, scale):
     w = workloads.Workload(f"scale_{scale}_{head_dim}", 3, head_dim, tuple(reqs), 23)
     run = pu.GpuRun(w, mode="beyond", kernel=kernel, scale=scale)
     pu.full_compare(run)
+
+
+@pytest.mark.parametrize("head_dim", [64, 128])
+def test_layers_keep_their_own_cache(head_dim):
+    """Four layers of one cache built from layer-specific inputs (in the order
+    2, 0, 3, 1), then one step of every layer: each step is compared with the
+    oracle on that layer's own static and live inputs, and each slot holds
+    that layer's reference K/V bit for bit."""
+    rng = np.random.default_rng(40 + head_dim)
+    reqs = list(workloads.random_requests(rng, 3, max_len=400))
+    w = workloads.Workload(f"layers_{head_dim}", 3, head_dim, tuple(reqs), 29)
+    seg = rcb.Segments.from_workload(w)
+    H, D = w.num_heads, w.head_dim
+    rcb.set_kernel("tcgen05")
+    cache = rcb.RefCache(seg, num_layers=4)
+    static = {l: workloads.static_qkv(w, l) for l in range(4)}
+    live = {l: workloads.live_qkv(w, l, step=l) for l in range(4)}
+    for l in (2, 0, 3, 1):
+        o = torch.empty(seg.static_rows, H, D, dtype=torch.bfloat16, device="cuda")
+        cache.build(l, *(t.cuda() for t in static[l]), o)
+    outs = {}
+    for l in range(4):
+        outs[l] = torch.full((seg.live_rows, H, D), float("nan"), dtype=torch.bfloat16, device="cuda")
+        cache.step(l, *(t.cuda() for t in live[l]), outs[l])
+    torch.cuda.synchronize()
+    assert rcb.status() == rcb.OK
+    scale = 1.0 / np.sqrt(D)
+    coff = pu.cache_offsets(w, "beyond")
+    for l in range(4):
+        k_slot, v_slot = (pu.bits(t) for t in cache.kv(l))
+        o = pu.f64(outs[l])
+        for b, r in enumerate(w.requests):
+            ref, _ = pu.oracle_live_request(w, "beyond", b, static[l], live[l], scale)
+            l0 = w.cu_live[b]
+            err = np.abs(o[l0:l0 + r.n_live] - ref)
+            assert err.size == 0 or (err.max() <= pu.MAX_ABS and err.mean() <= pu.MEAN_ABS), (l, b)
+            s0 = w.cu_static[b]
+            k_ref = pu.bits(static[l][1])[s0 + r.n_st:s0 + r.n_static]
+            v_ref = pu.bits(static[l][2])[s0 + r.n_st:s0 + r.n_static]
+            assert np.array_equal(k_slot[coff[b]:coff[b + 1]], k_ref) and np.array_equal(v_slot[coff[b]:coff[b + 1]], v_ref), (l, b)
