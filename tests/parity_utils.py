@@ -95,7 +95,7 @@ def full_compare(run: GpuRun, scale=None):
     """Every output row of both calls against the oracle (at the run's softmax
     scale unless one is given)."""
     w, mode = run.w, run.mode
-    scale = scale or run.scale or 1.0 / math.sqrt(w.head_dim)
+    scale = scale or getattr(run, "scale", None) or 1.0 / math.sqrt(w.head_dim)
     o_s, l_s, o_l, l_l = f64(run.o_static), f64(run.lse_static), f64(run.o_live), f64(run.lse_live)
     coff = cache_offsets(w, mode)
     for b, r in enumerate(w.requests):
