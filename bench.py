@@ -352,9 +352,11 @@ def run_ours(args, ws, rank, local):
         },
         "roofline": {
             "kernel": ("attn_mma_kernel (mma.sync)" if args.kernel == "mma_sync" else
-                       "attn_tc2_kernel (tcgen05, CTA pairs, 128-key tiles)" if D == 128 and args.kernel == "tcgen05_k128"
-                       else "attn_tc2_kernel (tcgen05, CTA pairs, 192-key tiles)" if D == 128
-                       else "attn_tc_kernel<64> (tcgen05)") + " in step_attention",
+                       "attn_tc2_kernel (tcgen05, CTA pairs, 128-key tiles"
+                       + (")" if D == 128 else ", head dim 64 padded to 128)")
+                       if args.kernel == "tcgen05_k128" or args.cache == "fp8"
+                       else "attn_tc2_kernel (tcgen05, CTA pairs, 192-key tiles"
+                       + (")" if D == 128 else ", head dim 64 padded to 128)")) + " in step_attention",
             "bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
             "frac": achieved / peak,
             "peak_kind": (f"bf16 dense, {pk['source']} burst (the timed region runs near the maximum SM clock)"

@@ -41,14 +41,14 @@
  *   - Host arrays (segment tables) are read during the call only; the library
  *     keeps its own copies.
  *   - No entry point allocates device memory except refcache_create (the
- *     cache, unless it is given memory, and for head_dim 128 a separate work
+ *     cache, unless it is given memory, and a separate work
  *     list with a workspace for split items, see refcache_create) and
  *     full_attention (a per-device work-list buffer that it keeps and grows).
  *   - The refcache_build, refcache_build_in_slot and step_attention calls of
  *     one cache share that workspace and the cache's work counter: issue them
  *     in stream order (one stream, or streams ordered by events), not
  *     concurrently.  Calls for different caches may run concurrently.
- *   - The head-dim-128 attention kernel and the merge of split items are
+ *   - The tcgen05 attention kernel and the merge of split items are
  *     launched as programmatic dependents of the previous kernel on the
  *     stream: they wait for it to complete before they read memory, and they
  *     allow the kernel after them to start early.  A caller's kernel launched
@@ -114,10 +114,11 @@ extern "C" {
 #define REFCACHE_CACHE_FP8 0x100
 
 /* Kernel selection (refcache_set_kernel): the tcgen05/TMEM/TMA kernel is the
- * default (at head_dim 128 on CTA pairs with 192-key tiles for the bf16
- * cache); the mma.sync kernel is the recompiled legacy-tensor-core baseline;
+ * default (on CTA pairs with 192-key tiles for the bf16 cache; head_dim 64
+ * runs on the same kernel with the head dim padded to 128 inside shared
+ * memory); the mma.sync kernel is the recompiled legacy-tensor-core baseline;
  * TCGEN05_K128 is the same tcgen05 pair kernel with 128-key tiles, kept as a
- * comparison point (head_dim 64 and the E4M3 cache always use 128-key tiles). */
+ * comparison point (the E4M3 cache always uses 128-key tiles). */
 #define REFCACHE_KERNEL_TCGEN05 0
 #define REFCACHE_KERNEL_MMA_SYNC 1
 #define REFCACHE_KERNEL_TCGEN05_K128 2
@@ -161,7 +162,7 @@ REFCACHE_API size_t refcache_bytes(int num_layers, int mask_mode, const refcache
  * otherwise it uses dev_mem (>= refcache_bytes(), 256-byte aligned, owned by
  * the caller, not freed).  Synchronous.  *out is set only on success.
  *
- * For head_dim 128 it also plans, for the current device, the per-item work
+ * It also plans, for the current device, the per-item work
  * lists of the prefill and the step, (query tile, head) items longest first;
  * a launch hands them out in that order to whichever CTA pair is free,
  * through a work counter kept in the cache's memory (reset by the launch
@@ -290,12 +291,10 @@ REFCACHE_API int full_attention(int batch, int num_heads, int head_dim, const in
  * nothing: no cudaMalloc, no cudaFree, no allocating library routine.  The
  * caller still passes (and owns) q, k, v, o and lse.
  *   - The array holds REFCACHE_NOALLOC_MAX_TASKS work items (512 KiB).  One
- *     item covers up to 128 query rows of a request at head_dim 64 and up to
- *     256 at head_dim 128, so a request of n rows needs ceil(n / 128) items at
- *     head_dim 64 and ceil(n / 256) at head_dim 128: at most 16384 x 128 rows
- *     per call at head_dim 64, 16384 x 256 at head_dim 128 (fewer when
- *     requests end mid-item).  Larger inputs are rejected with
- *     REFCACHE_ERR_INVALID_ARG and a message naming the limit.
+ *     item covers up to 256 query rows of a request (either head_dim), so a
+ *     request of n rows needs ceil(n / 256) items: at most 16384 x 256 rows
+ *     per call (fewer when requests end mid-item).  Larger inputs are
+ *     rejected with REFCACHE_ERR_INVALID_ARG and a message naming the limit.
  *   - The first call on each device looks up the array's device address with
  *     that device current (a one-time set-up).
  *   - Every call rewrites the whole work list it uses, so no state carries

@@ -1,6 +1,9 @@
-// attn_tc2.cuh -- the head_dim-128 attention kernel on CTA pairs: the same
-// computation and pair schedule as attn_tc.cuh, with every MMA issued over
-// two CTAs on neighbouring SMs (tcgen05 cta_group::2, M = 256).
+// attn_tc2.cuh -- the tcgen05 attention kernel on CTA pairs: for every
+// (task, head) item, O = softmax(scale * Q K^T) V over the task's visible keys
+// (key ranges A then B; see common.cuh), scores, softmax and accumulation in
+// fp32 and P rounded to bf16 for P.V, with every MMA issued over two CTAs on
+// neighbouring SMs (tcgen05 cta_group::2, M = 256).  Head dim 128, or 64
+// padded to 128 inside shared memory (see the kernel's kDG).
 //
 // Why pairs: with one 128-row query tile per SM, each S/P.V pair of MMAs
 // (1024 tensor cycles at 128-key tiles) needs a fresh 32 KB K tile and 32 KB
@@ -162,8 +165,9 @@ struct SmemT {
   static constexpr uint32_t kAbort = kTmemHolder + 4;
   // load record of each CTA of the pair (leader's copy read at teardown):
   // per CTA [loads per stage (kStages) | own bytes of the last load per stage
-  // (kStages) | loads per Q buffer (2)]
-  static constexpr uint32_t kRecWords = 2 * kStages + 2;
+  // (kStages) | the other CTA's bytes of that load (kStages) | loads per Q
+  // buffer (2)]
+  static constexpr uint32_t kRecWords = 3 * kStages + 2;
   static constexpr uint32_t kLoadRec = kAbort + 4;
   // ring of taken items (work counter): slot k % kItemSlots holds item k of
   // this cluster (-1: none left); the gate warp passes the MMA warp its item
@@ -238,7 +242,13 @@ __device__ __forceinline__ void work_done(int* work, int n_clusters) {
 }
 }  // namespace tc2
 
-template <bool kF8, int kBN>
+// kDG: the tensors' head dim.  At 64 the tiles keep the layout of head dim
+// 128 with the upper 64 columns as zero padding: Q and K tiles load only
+// their first 64-column box (S = Q K^T takes the first four K = 16 steps), the
+// second CTA of a pair holds the upper half of V's columns, which it never
+// loads but zeroes once (P V keeps N = 128; O's upper 64 columns stay zero and
+// are never read).
+template <bool kF8, int kBN, int kDG>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::kThreads, 1)
     attn_tc2_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_ka,
                     const __grid_constant__ CUtensorMap tm_va, const __grid_constant__ CUtensorMap tm_kb,
@@ -259,7 +269,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
   using tc2::kKHalf8;
   using tc2::kVHalf8;
   using L = tc2::SmemT<kF8, kBN>;
-  constexpr int D = tc2::kD;
+  constexpr int D = tc2::kD;   // head-dim columns of the tiles (P V's N)
+  constexpr int DG = kDG;      // head dim of the tensors
+  static_assert(DG == D || (DG == 64 && !kF8), "head dim 128, or 64 (bf16 cache) padded to 128");
+  constexpr int kQBoxes = DG / 64;  // 64-column boxes of a Q or K row loaded
   auto stage_of = [](int g) -> int { return tc2::stage_of<kStages>(g); };
   auto stage_parity = [](int g) -> uint32_t { return tc2::stage_parity<kStages>(g); };
   constexpr uint32_t kIdescS = idesc_bf16_f32(256, kBN, false);
@@ -309,6 +322,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
     *abort_flag = 0;
     fence_barrier_init();
     fence_proxy_async_smem();
+  }
+  if constexpr (DG != D) {
+    // head dim 64: the second CTA's V half of every stage is the zero padding
+    // of the upper 64 head-dim columns (written once; that CTA never loads V)
+    if (rank == 1) {
+      constexpr uint32_t kChunks = kVHalf / 16;
+      for (uint32_t i = threadIdx.x; i < kStages * kChunks; i += blockDim.x)
+        st_shared_v4(base + L::kRing + (i / kChunks) * kStage + kKHalf + (i % kChunks) * 16u, make_uint4(0, 0, 0, 0));
+      fence_proxy_async_smem();
+    }
   }
   if (warp == Cfg::kMmaWarp) {
     tmem_alloc_pair(smem_u32(tmem_holder), kTmemCols);
@@ -373,10 +396,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
       // last load of each stage; the leader arms every phase for both CTAs'
       // bytes right before it issues its own half
       int n_stage[kStages];
-      uint32_t own_bytes[kStages];
+      uint32_t own_bytes[kStages], other_bytes[kStages];
       for (int s = 0; s < kStages; ++s) {
         n_stage[s] = 0;
         own_bytes[s] = 0;
+        other_bytes[s] = 0;
       }
       int n_q[2] = {0, 0};
       int scale_armed[tc2::kScaleSlots];
@@ -397,8 +421,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
         const TileSrc ks = tc2::tile_src<kBN>(tk, na, kj >= 0 ? kj : 0);
         const TileSrc vs = tc2::tile_src<kBN>(tk, na, vj >= 0 ? vj : 0);
         const bool k8 = kF8 && kj >= 0 && ks.in_b, v8 = kF8 && vj >= 0 && vs.in_b;
-        const uint32_t bytes =
-            2 * ((kj >= 0 ? (k8 ? kKHalf8 : kKHalf) : 0u) + (vj >= 0 ? (v8 ? kVHalf8 : kVHalf) : 0u));
+        // each CTA's K bytes; a V half (at head dim 64 only the first CTA loads one)
+        const uint32_t kb = kj >= 0 ? (k8 ? kKHalf8 : kKBox * kQBoxes) : 0u;
+        const uint32_t vb = vj >= 0 ? (v8 ? kVHalf8 : kVHalf) : 0u;
+        const bool v_here = DG == D || rank == 0;
+        const uint32_t bytes = 2 * kb + (DG == D ? 2 : 1) * vb;  // both CTAs
         if (k8) {
           // this CTA's softmax warps read the cached tile's scales from ring slot
           // si % kScaleSlots; the slot's previous tile must have been read
@@ -416,20 +443,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
         } else {
           if (leader) mbar_arrive_expect_tx(bar(L::kStageFull + slot), bytes);
           ++n_stage[slot];
-          own_bytes[slot] = bytes / 2;
+          own_bytes[slot] = kb + (v_here ? vb : 0u);
+          other_bytes[slot] = kb + (DG == D || rank == 1 ? vb : 0u);
           if (k8) {  // E4M3 keys [64 r, 64 r + 64): one box of 64 rows x 128 bytes
             tma_load_2d_pair(dst, &tm_kb, full, head * D, ks.row + 64 * static_cast<int>(rank));
           } else if (kj >= 0) {  // keys [kBN/2 r, kBN/2 (r + 1)) of the tile, both head-dim boxes
             const void* map = ks.in_b ? &tm_kb : &tm_ka;
-            for (int ch = 0; ch < 2; ++ch)
-              tma_load_2d_pair(dst + ch * kKBox, map, full, head * D + ch * 64,
+            for (int ch = 0; ch < kQBoxes; ++ch)
+              tma_load_2d_pair(dst + ch * kKBox, map, full, head * DG + ch * 64,
                                ks.row + (kBN / 2) * static_cast<int>(rank));
           }
           if (v8) {  // E4M3 V^T rows d in [64 r, 64 r + 64), all 128 keys
             tma_load_2d_pair(dst + kKHalf, &tm_vb, full, vs.row, head * D + 64 * static_cast<int>(rank));
-          } else if (vj >= 0) {  // head-dim columns [64 r, 64 r + 64) of all kBN keys
+          } else if (vj >= 0 && v_here) {  // head-dim columns [64 r, 64 r + 64) of all kBN keys
             const void* map = vs.in_b ? &tm_vb : &tm_va;
-            tma_load_2d_pair(dst + kKHalf, map, full, head * D + 64 * static_cast<int>(rank), vs.row);
+            tma_load_2d_pair(dst + kKHalf, map, full, head * DG + 64 * static_cast<int>(rank), vs.row);
           }
         }
         ++g;
@@ -446,11 +474,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
           const int b = qi & 1;
           const uint32_t n = static_cast<uint32_t>(qi >> 1);
           if (!wait_one(bar(L::kQEmpty + b), (n & 1u) ^ 1u, ctl, 1)) goto producer_done;
-          if (leader) mbar_arrive_expect_tx(bar(L::kQFull + b), 2 * kQTile);
+          if (leader) mbar_arrive_expect_tx(bar(L::kQFull + b), 2 * kQBoxes * kBoxBytes);
           ++n_q[b];
           const uint32_t qfull = lbar(L::kQFull + b);
-          for (int ch = 0; ch < 2; ++ch)
-            tma_load_2d_pair(base + L::kQ + b * kQTile + ch * kBoxBytes, &tm_q, qfull, head * D + ch * 64,
+          for (int ch = 0; ch < kQBoxes; ++ch)
+            tma_load_2d_pair(base + L::kQ + b * kQTile + ch * kBoxBytes, &tm_q, qfull, head * DG + ch * 64,
                              tk.q_row0 + 128 * static_cast<int>(rank));
         }
         if (!load_stage(0, -1)) goto producer_done;
@@ -470,9 +498,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
       for (int s = 0; s < kStages; ++s) {
         st_cluster_u32(rec + 4u * s, static_cast<uint32_t>(n_stage[s]));
         st_cluster_u32(rec + 4u * (kStages + s), own_bytes[s]);
+        st_cluster_u32(rec + 4u * (2 * kStages + s), other_bytes[s]);
       }
-      st_cluster_u32(rec + 4u * (2 * kStages), static_cast<uint32_t>(n_q[0]));
-      st_cluster_u32(rec + 4u * (2 * kStages + 1), static_cast<uint32_t>(n_q[1]));
+      st_cluster_u32(rec + 4u * (3 * kStages), static_cast<uint32_t>(n_q[0]));
+      st_cluster_u32(rec + 4u * (3 * kStages + 1), static_cast<uint32_t>(n_q[1]));
     }
     __syncwarp();
   } else if (warp == Cfg::kMmaWarp) {
@@ -521,7 +550,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
                   tc2_mma_ss_f8(d_s, q8d + ((32u * kk) >> 4), kd + ((32u * kk) >> 4), kIdesc8, kk > 0 ? 1u : 0u);
               } else {
 #pragma unroll
-                for (int kk = 0; kk < D / 16; ++kk)
+                for (int kk = 0; kk < DG / 16; ++kk)
                   tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
               }
               if (n == nkv - 1) tc2_commit_mc(bar(L::kQEmpty + qb), 3);
@@ -555,13 +584,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
                 for (int kk = 0; kk < kBN / 16; ++kk)
                   tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, kk > 0 ? 1u : acc0);
 #pragma unroll
-                for (int kk = 0; kk < D / 16; ++kk)
+                for (int kk = 0; kk < DG / 16; ++kk)
                   tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
               } else if (!s8) {
 #pragma unroll
                 for (int kk = 0; kk < 8; ++kk) {
                   tc2_mma_ts(tmem + kColO, a_p + 8u * kk, vd + ((2048u * kk) >> 4), kIdescO, kk > 0 ? 1u : acc0);
-                  tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
+                  if (kk < DG / 16) tc2_mma_ss(d_s, qd + q_off(kk), kd + k_off(kk), kIdescS, kk > 0 ? 1u : 0u);
                 }
               } else if (pv8) {
 #pragma unroll
@@ -653,7 +682,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
     // epilogue through shared memory.
     constexpr int kH = Cfg::kHalves;
     constexpr int kC = kBN / kH;  // key columns of this thread
-    constexpr int kOC = D / kH;   // O columns of this thread
+    constexpr int kOC = DG / kH;  // O columns of this thread
     const int quarter = warp & 3, hh = warp >> 2;
     const int col0 = hh * kC, ocol0 = hh * kOC;
     const int trow = quarter * 32 + lane;                  // row within this CTA's 128 rows (= TMEM lane)
@@ -681,7 +710,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
       const int nkv = tc2::n_key_tiles<kBN>(tk, na);
       const bool row_ok = prow < tk.q_rows;
       const int64_t grow = static_cast<int64_t>(tk.q_row0) + prow;
-      __nv_bfloat16* orow = args.out + grow * args.row_stride + static_cast<int64_t>(head) * D + ocol0;
+      __nv_bfloat16* orow = args.out + grow * args.row_stride + static_cast<int64_t>(head) * DG + ocol0;
       if (nkv == 0) {
         if (row_ok) {
           uint4 z = make_uint4(0, 0, 0, 0);
@@ -952,7 +981,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
           decode_item(args, item, et, e_head);
           e_row_ok = prow < et.q_rows;
           e_grow = static_cast<int64_t>(et.q_row0) + prow;
-          e_orow = args.out + e_grow * args.row_stride + static_cast<int64_t>(e_head) * D + ocol0;
+          e_orow = args.out + e_grow * args.row_stride + static_cast<int64_t>(e_head) * DG + ocol0;
           e_part = et.part;
         }
         if (!wait_group(G + nkv + 1, 10)) goto softmax_done;  // the item's last group
@@ -972,7 +1001,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
         if (e_part > 0) {
           // a part of a split item: O / l in fp32 and m + log l to its workspace slot
           const int64_t prow_ws = static_cast<int64_t>(e_part - 1) * args.rows_per_task + prow;
-          float4* dst = reinterpret_cast<float4*>(args.part_o + prow_ws * D + ocol0);
+          float4* dst = reinterpret_cast<float4*>(args.part_o + prow_ws * DG + ocol0);
 #pragma unroll
           for (int cc = 0; cc < kOC / 32; ++cc) {
             uint32_t o[32];
@@ -1038,21 +1067,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(tc2::Cfg<kF8, kBN>::
     // arrived.  Then the last phase of every barrier is drained (bounded).
     const volatile uint32_t* rec = reinterpret_cast<const volatile uint32_t*>(base_ptr + L::kLoadRec);
     const volatile uint32_t* peer = rec + L::kRecWords;
-    auto settle = [&](uint32_t b, int mine, int theirs, uint32_t mine_bytes, uint32_t their_bytes) {
+    // missing: the follower's bytes of the leader's last phase; loaded: the
+    // follower's own bytes of its last load
+    auto settle = [&](uint32_t b, int mine, int theirs, uint32_t missing, uint32_t loaded) {
       if (theirs == mine + 1) {
-        mbar_arrive_expect_tx(b, their_bytes);
+        mbar_arrive_expect_tx(b, loaded);
         mine = theirs;
-      } else if (mine == theirs + 1 && mine_bytes > 0) {
-        mbar_complete_tx(b, mine_bytes);
+      } else if (mine == theirs + 1 && missing > 0) {
+        mbar_complete_tx(b, missing);
       }
       if (mine > 0) drain_one(b, static_cast<uint32_t>(mine - 1) & 1u, args.timeout_ns);
     };
     for (int s = 0; s < kStages; ++s)
-      settle(bar(L::kStageFull + s), static_cast<int>(rec[s]), static_cast<int>(peer[s]), rec[kStages + s],
+      settle(bar(L::kStageFull + s), static_cast<int>(rec[s]), static_cast<int>(peer[s]), rec[2 * kStages + s],
              peer[kStages + s]);
+    constexpr uint32_t kQCta = kQBoxes * kBoxBytes;  // each CTA's bytes of a Q load
     for (int b = 0; b < 2; ++b)
-      settle(bar(L::kQFull + b), static_cast<int>(rec[2 * kStages + b]), static_cast<int>(peer[2 * kStages + b]),
-             kQTile, kQTile);
+      settle(bar(L::kQFull + b), static_cast<int>(rec[3 * kStages + b]), static_cast<int>(peer[3 * kStages + b]),
+             kQCta, kQCta);
   }
   // the follower leaves only once the leader has seen every load of the pair land
   cluster_sync();

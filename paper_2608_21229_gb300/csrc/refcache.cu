@@ -1,10 +1,10 @@
 // refcache.cu -- the C ABI declared in include/refcache.h: argument checks,
 // the per-request work tables, the persistent per-layer K/V cache (bf16, or
 // E4M3 with REFCACHE_CACHE_FP8), TMA tensor maps and the kernel launches.  All
-// compute runs in the kernels of attn_tc2.cuh (head dim 128, CTA pairs),
-// attn_tc.cuh (head dim 64), attn_mma.cuh (the mma.sync comparison kernel and
-// the cache copy), attn_combine.cuh (merge of split items) and cache_fp8.cuh
-// (the E4M3 cache write).
+// compute runs in the kernels of attn_tc2.cuh (the tcgen05 kernel on CTA
+// pairs, both head dims; attn_tc.cuh holds its bounded waits), attn_mma.cuh
+// (the mma.sync comparison kernel and the cache copy), attn_combine.cuh (merge
+// of split items) and cache_fp8.cuh (the E4M3 cache write).
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -61,8 +61,8 @@ struct DeviceInfo {
   bool checked = false;
   bool ok = false;
   int num_sms = 0;
-  bool attr_set[7] = {false, false, false, false, false, false, false};
-  int max_clusters[3] = {0, 0, 0};  // CTA pairs of each attn_tc2_kernel variant that fit at once
+  bool attr_set[9] = {false, false, false, false, false, false, false, false, false};
+  int max_clusters[5] = {0, 0, 0, 0, 0};  // CTA pairs of each attn_tc2_kernel variant that fit at once
 };
 DeviceInfo g_dev[kMaxDevices];
 std::mutex g_dev_mu;
@@ -147,9 +147,8 @@ int make_tmap_u8(CUtensorMap* m, const void* base, int64_t inner, int64_t outer)
 }
 
 // ---------------------------------------------------------------- work lists
-// Query rows per task: one M = 256 MMA of a CTA pair for head_dim 128, one
-// 128-row tile of a single CTA for head_dim 64.
-int task_rows(int D) { return D == 128 ? 256 : 128; }
+// Query rows per task: one M = 256 MMA of a CTA pair (both head dims).
+int task_rows(int) { return 256; }
 
 void add_rows(std::vector<Task>& v, int rows_per_task, int q0, int qn, int a0, int an, int b0, int bn) {
   for (int r = 0; r < qn; r += rows_per_task) {
@@ -200,45 +199,29 @@ int check_scale(float s) {
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // ---------------------------------------------------------------- launches
-template <int D>
-int launch_tc(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info, cudaStream_t s) {
-  constexpr uint32_t smem = rc::tc::Smem<D>::kDynamic;
-  const int key = D == 64 ? 0 : 1;
-  if (!info->attr_set[key]) {
-    cudaError_t e = cudaFuncSetAttribute(rc::attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_tc_kernel)");
-    info->attr_set[key] = true;
-  }
-  const int grid = std::min(a.n_items, info->num_sms);
-  rc::attn_tc_kernel<D><<<grid, rc::tc::kThreads, smem, s>>>(maps[0], maps[1], maps[2], maps[3], maps[4], a);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return cuda_fail(e, "attn_tc_kernel launch");
-  return REFCACHE_OK;
-}
-
-// Keys per tile of the head-dim-128 pair kernel: 192 for the bf16 cache
+// Keys per tile of the pair kernel: 192 for the bf16 cache
 // (REFCACHE_KERNEL_TCGEN05), 128 for the E4M3 cache and for
 // REFCACHE_KERNEL_TCGEN05_K128.
 int tc2_tile(bool f8) { return f8 || g_kernel.load() == REFCACHE_KERNEL_TCGEN05_K128 ? 128 : 192; }
 
-// CTA pairs of the head-dim-128 kernel (bf16 key range B, or E4M3 with kF8;
-// kBN keys per tile) that run at once on this device (the persistent grid);
-// sets the kernel's shared-memory attribute on first use.
-template <bool kF8, int kBN>
+// CTA pairs of the pair kernel (bf16 key range B, or E4M3 with kF8; kBN keys
+// per tile; head dim kDG) that run at once on this device (the persistent
+// grid); sets the kernel's shared-memory attribute on first use.
+template <bool kF8, int kBN, int kDG>
 int tc2_clusters(DeviceInfo* info, int* clusters_out) {
   constexpr uint32_t smem = rc::tc2::SmemT<kF8, kBN>::kDynamic;
-  const int variant = kF8 ? 1 : kBN == 128 ? 0 : 2;
+  const int variant = kF8 ? 1 : kDG == 128 ? (kBN == 128 ? 0 : 2) : (kBN == 128 ? 3 : 4);
   const int key = 4 + variant;
   if (!info->attr_set[key]) {
     cudaError_t e =
-        cudaFuncSetAttribute(rc::attn_tc2_kernel<kF8, kBN>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        cudaFuncSetAttribute(rc::attn_tc2_kernel<kF8, kBN, kDG>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(attn_tc2_kernel)");
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3(2 * static_cast<unsigned>(info->num_sms / 2), 1, 1);
     cfg.blockDim = dim3(rc::tc2::Cfg<kF8, kBN>::kThreads, 1, 1);
     cfg.dynamicSmemBytes = smem;
     int clusters = 0;
-    e = cudaOccupancyMaxActiveClusters(&clusters, rc::attn_tc2_kernel<kF8, kBN>, &cfg);
+    e = cudaOccupancyMaxActiveClusters(&clusters, rc::attn_tc2_kernel<kF8, kBN, kDG>, &cfg);
     if (e != cudaSuccess || clusters < 1) clusters = info->num_sms / 2;
     info->max_clusters[variant] = clusters;
     info->attr_set[key] = true;
@@ -247,12 +230,12 @@ int tc2_clusters(DeviceInfo* info, int* clusters_out) {
   return REFCACHE_OK;
 }
 
-// The CTA-pair kernel (head_dim 128): grid = 2 x the clusters that fit at once.
-template <bool kF8, int kBN>
+// The CTA-pair kernel: grid = 2 x the clusters that fit at once.
+template <bool kF8, int kBN, int kDG>
 int launch_tc2(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info, cudaStream_t s) {
   constexpr uint32_t smem = rc::tc2::SmemT<kF8, kBN>::kDynamic;
   int max_clusters = 0;
-  int rc = tc2_clusters<kF8, kBN>(info, &max_clusters);
+  int rc = tc2_clusters<kF8, kBN, kDG>(info, &max_clusters);
   if (rc) return rc;
   const int clusters = std::min(a.n_items, max_clusters);
   // a programmatic dependent of the stream's previous kernel: its prologue
@@ -268,7 +251,7 @@ int launch_tc2(const CUtensorMap (&maps)[5], const AttnArgs& a, DeviceInfo* info
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   cudaError_t e =
-      cudaLaunchKernelEx(&cfg, rc::attn_tc2_kernel<kF8, kBN>, maps[0], maps[1], maps[2], maps[3], maps[4], a);
+      cudaLaunchKernelEx(&cfg, rc::attn_tc2_kernel<kF8, kBN, kDG>, maps[0], maps[1], maps[2], maps[3], maps[4], a);
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "attn_tc2_kernel launch");
   return REFCACHE_OK;
@@ -311,7 +294,7 @@ struct Fp8B {
   int64_t rows_pad = 0;
 };
 
-// A per-item work list with split items (head-dim-128 tcgen05 kernel only):
+// A per-item work list with split items (tcgen05 kernel only):
 // the items, the combine jobs of the split ones and their workspace.
 struct ItemList {
   const Task* items = nullptr;
@@ -356,8 +339,8 @@ int launch_copy(const CopyJob& c, const DeviceInfo* info, cudaStream_t s, bool b
   return REFCACHE_OK;
 }
 
-// `copy` (the build's cache write, if any) runs beside the head-dim-128 pair
-// kernel, launched right after it; with the other kernels it goes first.
+// `copy` (the build's cache write, if any) runs beside the pair kernel,
+// launched right after it; with the mma.sync kernel it goes first.
 int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands& op, float scale, DeviceInfo* info,
                   cudaStream_t s, const ItemList* il = nullptr, const Fp8B* f8 = nullptr,
                   const CopyJob* copy = nullptr) {
@@ -387,11 +370,11 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
     if (rc) return rc;
     return D == 64 ? launch_mma<64>(a, info, s) : launch_mma<128>(a, info, s);
   }
-  // Key tiles of the CTA-pair kernel: each CTA loads half of a K tile (two
-  // boxes of tile / 2 rows) and a V box of the whole tile; head dim 64 loads
-  // 128-row boxes.
-  const uint32_t tile = D == 128 ? static_cast<uint32_t>(tc2_tile(f8 != nullptr)) : 128u;
-  const uint32_t k_rows = D == 128 ? tile / 2 : 128u, v_rows = tile;
+  // Key tiles of the CTA-pair kernel: each CTA loads half of a K tile (boxes
+  // of tile / 2 rows, one per 64 head-dim columns) and a V box of the whole
+  // tile.
+  const uint32_t tile = static_cast<uint32_t>(tc2_tile(f8 != nullptr));
+  const uint32_t k_rows = tile / 2, v_rows = tile;
   CUtensorMap maps[5];
   int rc;
   if ((rc = make_tmap(&maps[0], op.q, op.q_rows, H, D)) != 0) return rc;
@@ -409,10 +392,6 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
     maps[4] = maps[2];
   }
   a.dbg_skip_first_load = g_dbg_skip.exchange(0);
-  if (D == 64) {
-    if (copy && (rc = launch_copy(*copy, info, s, false)) != 0) return rc;
-    return launch_tc<64>(maps, a, info, s);
-  }
   if (il && il->items) {
     a.tasks = il->items;
     a.per_item = 1;
@@ -420,8 +399,12 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
     a.part_o = il->part_o;
     a.part_lse = il->part_lse;
   }
-  rc = f8 ? launch_tc2<true, 128>(maps, a, info, s)
-          : tile == 128 ? launch_tc2<false, 128>(maps, a, info, s) : launch_tc2<false, 192>(maps, a, info, s);
+  if (f8)
+    rc = launch_tc2<true, 128, 128>(maps, a, info, s);
+  else if (D == 128)
+    rc = tile == 128 ? launch_tc2<false, 128, 128>(maps, a, info, s) : launch_tc2<false, 192, 128>(maps, a, info, s);
+  else
+    rc = tile == 128 ? launch_tc2<false, 128, 64>(maps, a, info, s) : launch_tc2<false, 192, 64>(maps, a, info, s);
   if (rc) return rc;
   if (copy && (rc = launch_copy(*copy, info, s, true)) != 0) return rc;
   if (il && il->n_jobs > 0) {
@@ -434,9 +417,12 @@ int run_attention(const Task* d_tasks, int n_tasks, int H, int D, const Operands
     attr[0].val.programmaticStreamSerializationAllowed = 1;  // its CTAs wait for the attention kernel
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, rc::combine_parts_kernel<128>, il->jobs,
-                                       static_cast<const float*>(il->part_o), static_cast<const float*>(il->part_lse),
-                                       a.rows_per_task, a.out, a.lse, a.row_stride, H);
+    const float* po = static_cast<const float*>(il->part_o);
+    const float* pl = static_cast<const float*>(il->part_lse);
+    cudaError_t e = D == 128 ? cudaLaunchKernelEx(&cfg, rc::combine_parts_kernel<128>, il->jobs, po, pl, a.rows_per_task,
+                                                  a.out, a.lse, a.row_stride, H)
+                             : cudaLaunchKernelEx(&cfg, rc::combine_parts_kernel<64>, il->jobs, po, pl, a.rows_per_task,
+                                                  a.out, a.lse, a.row_stride, H);
     if (e == cudaSuccess) e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "combine_parts_kernel launch");
   }
@@ -558,7 +544,7 @@ struct refcache {
   int n_step = 0;
   CopySeg* d_copy = nullptr;
   int n_copy = 0;
-  // per-item lists of the head-dim-128 kernel, ordered for the persistent
+  // per-item lists of the pair kernel, ordered for the persistent
   // grid (the step's with split items), in a separate allocation:
   // [build items | step items | step jobs | part_o | part_lse]
   uint8_t* aux = nullptr;
@@ -727,7 +713,7 @@ int check_ptrs(std::initializer_list<const void*> ps, int64_t rows, const char* 
   return REFCACHE_OK;
 }
 
-// Per-item lists of a head-dim-128 handle for the current device, in one
+// Per-item lists of a handle for the current device, in one
 // allocation of their own (the caller-sized cache memory is not touched):
 // the step's, with the last round of items split, and the prefill's, whose
 // items are never split: each runs whole on one CTA pair, so a request's
@@ -741,8 +727,9 @@ int plan_split_items(refcache* h, DeviceInfo* info, const std::vector<Task>& bt,
   const bool f8 = h->f8 && h->rows_pad > 0;
   const int tile = tc2_tile(f8), tile_b = tc2_tile(false);
   int clusters = 0;
-  int rc = f8 ? tc2_clusters<true, 128>(info, &clusters)
-              : tile == 128 ? tc2_clusters<false, 128>(info, &clusters) : tc2_clusters<false, 192>(info, &clusters);
+  int rc = f8 ? tc2_clusters<true, 128, 128>(info, &clusters)
+              : tile == 128 ? tc2_clusters<false, 128, 128>(info, &clusters)
+                            : tc2_clusters<false, 192, 128>(info, &clusters);
   if (rc) return rc;
   std::vector<Task> si, bi;
   std::vector<CombineJob> sj;
@@ -879,7 +866,7 @@ int refcache_create(refcache_t** out, int num_layers, int mask_mode, const refca
     delete h;
     return cuda_fail(e, "cudaMemcpy(work tables)");
   }
-  if (h->D == 128 && (rc = plan_split_items(h, info, bt, st)) != 0) {
+  if ((rc = plan_split_items(h, info, bt, st)) != 0) {
     if (h->owns) cudaFree(h->mem);
     delete h;
     return rc;

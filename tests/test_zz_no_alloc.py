@@ -77,13 +77,19 @@ def test_noalloc_matches_full_attention_twice(kernel, head_dim):
         rcb.set_kernel("tcgen05")
 
 
-@pytest.mark.parametrize("head_dim,rows_per_item", [(64, 128), (128, 256)])
-def test_noalloc_rejects_inputs_beyond_its_limit(head_dim, rows_per_item):
+@pytest.mark.parametrize("head_dim", [64, 128])
+def test_noalloc_rejects_inputs_beyond_its_limit(head_dim):
+    """One work item (256 query rows at either head dim) more than the static
+    array holds is refused.  The tensors are NULL, so that no kernel could run
+    even if the limit check let the call through (the pointer check would
+    refuse it next)."""
     lib = rcb.load()
-    rows = rcb.NOALLOC_MAX_TASKS * rows_per_item + 1  # one item more than the array holds
+    rows = rcb.NOALLOC_MAX_TASKS * 256 + 1
     cu = (ctypes.c_int32 * 2)(0, rows)
-    q = torch.empty(16, dtype=torch.bfloat16, device="cuda")
-    rc = lib.full_attention_noalloc(1, 1, head_dim, cu, q.data_ptr(), q.data_ptr(), q.data_ptr(), q.data_ptr(),
-                                    None, 0.125, None)
+    rc = lib.full_attention_noalloc(1, 1, head_dim, cu, None, None, None, None, None, 0.125, None)
     assert rc == rcb.ERR_INVALID_ARG
     assert "static limit" in rcb.last_error()
+    # exactly at the limit the same call passes the limit check and stops at the NULL pointers
+    cu_at = (ctypes.c_int32 * 2)(0, rcb.NOALLOC_MAX_TASKS * 256)
+    assert lib.full_attention_noalloc(1, 1, head_dim, cu_at, None, None, None, None, None, 0.125, None) == rcb.ERR_INVALID_ARG
+    assert "static limit" not in rcb.last_error()
